@@ -1,0 +1,376 @@
+#!/usr/bin/env python
+"""Throughput of the MoE expert layer, forward + backward, on GB300.
+
+A step is one pass of the whole layer (gating, aux loss, dispatch, expert FFN
+forward, combine, combine backward, expert FFN backward, gating backward,
+unpermute-reduce) over one batch of seeded synthetic tokens. The default workload
+is mid_bf16 (T=4096, d=1024, E=16 SwiGLU experts of F=2816, top-2, bf16 storage
+with fp32 accumulation).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+  python bench.py --impl reference ...   # the fp64 CPU oracle on the host cores
+
+Timing: W untimed warm-up steps, then K steps timed one by one with CUDA events on
+the launching stream; L2 is flushed (a 256 MiB write, outside the events) before
+every timed step. Under torchrun each rank runs its own replica (the layer does not
+shard; no collective on the data path); the time is the max over ranks and the
+value is the tokens of all ranks per second. Prints one JSON line on rank 0.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from synth import moe_inputs as mi  # noqa: E402
+
+METRIC = "MoE layer fwd+bwd tokens/s on 1 GB300"
+FLUSH_BYTES = 256 << 20
+
+
+def args_():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=300)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="mid_bf16")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-clocks", action="store_true")
+    return ap.parse_args()
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return {"hbm_gbs": p["hbm_gbs"], "bf16_tflops": p["bf16_tflops"],
+                "bf16_tflops_sustained": p.get("bf16_tflops_sustained"), "source": "measured"}
+    except Exception:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+                "source": "fallback"}
+
+
+def workload_desc(sh):
+    s = (f"{sh.name} (T={sh.T}, d={sh.d_model}, E={sh.n_experts}, F={sh.d_ff}, k={sh.top_k}"
+         f"{', P=%d' % sh.n_parties if sh.n_parties > 1 else ''}"
+         f"{', S=%d shared F=%d' % (sh.n_shared, sh.d_ff_shared) if sh.n_shared else ''})")
+    return s
+
+
+# --------------------------------------------------------------------------- memory bytes
+def mem_bytes_per_step(sh) -> float:
+    """Algorithmic HBM bytes of the memory-bound stages per step:
+    route read x + write logits/probs/picks; dispatch read x + write x_perm + tables;
+    combine read y_perm, w + write out; combine bwd read dout, y_perm + write dy, dw;
+    route bwd read probs, dw, x + write dlogits; unpermute read dx_perm (+ dlogits)
+    + write dx."""
+    b = 2 if sh.dtype == "bf16" else 4
+    T, d, E, k = sh.T, sh.d_model, sh.n_experts, sh.top_k
+    per_tok = 0.0
+    per_tok += d * b + 2 * E * 4 + k * 8                     # route
+    per_tok += d * b + k * d * b + 12 * k                    # dispatch
+    per_tok += k * d * b + k * 4 + d * b                     # combine fwd
+    per_tok += d * b + k * d * b + k * d * b + k * 4         # combine bwd
+    per_tok += 2 * E * 4 + k * 4 + d * b + E * 4             # route bwd
+    per_tok += k * d * b + E * 4 + d * b                     # unpermute-reduce
+    return per_tok * T
+
+
+# --------------------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int, enabled: bool = True):
+        self.proc = None
+        self.gpu = gpu_index
+        if enabled:
+            try:
+                self.proc = subprocess.Popen(
+                    ["nvidia-smi", "-i", str(gpu_index), f"--query-gpu={self.FIELDS}",
+                     "--format=csv,noheader,nounits", "-lms", "50"],
+                    stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            except Exception:
+                self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except Exception:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, mx, reasons = [], 0.0, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.strip().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx = max(mx, float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "samples": len(sm),
+                "reasons": sorted(reasons)}
+
+
+# --------------------------------------------------------------------------- traffic
+def gemm_traffic_record(sh):
+    """DRAM bytes per grouped-GEMM launch from the committed ncu summary, if it was
+    taken on the current kernel source (else None)."""
+    path = os.path.join(ROOT, "profiles", "gemm_traffic.json")
+    src = os.path.join(ROOT, "paper_2506_02965_gb300", "csrc", "gemm_tc.cu")
+    try:
+        rec = json.load(open(path))
+        h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        if rec.get("gemm_tc_sha") != h or rec.get("workload") != sh.name:
+            return None
+        return rec.get("dram_bytes_per_launch")
+    except Exception:
+        return None
+
+
+# --------------------------------------------------------------------------- oracle legs
+def oracle_sample(workload: str, tokens: int, repeats: int) -> dict:
+    """Time the fp64 oracle (fwd+bwd) on the first `tokens` tokens of the workload."""
+    import numpy as np
+
+    from oracle import moe_oracle as mo
+    sh = mi.shape_by_name(workload)
+    inp = mi.make_inputs(sh)
+    sub = {k: (np.asarray(v, np.float64) if isinstance(v, np.ndarray) and v.dtype == np.float32
+               else v) for k, v in inp.items()}
+    sub["x"] = sub["x"][:tokens]
+    sub["dout"] = sub["dout"][:tokens]
+    P = sh.n_parties
+    sub["party_offsets"] = (np.arange(P + 1) * (tokens // P)).astype(np.int32)
+    s2 = sh.with_(T=tokens - tokens % P)
+    times = []
+    for _ in range(repeats):
+        t0 = time.perf_counter()
+        f = mo.layer_forward(sub, s2)
+        mo.layer_backward(sub, s2, f)
+        times.append(time.perf_counter() - t0)
+    return {"tokens": s2.T, "seconds": times}
+
+
+def cpu_baseline(workload: str, tokens: int, repeats: int) -> dict:
+    """Run oracle_sample in a fresh interpreter with every host core for BLAS."""
+    cores = os.cpu_count() or 1
+    env = dict(os.environ, OPENBLAS_NUM_THREADS=str(cores), OMP_NUM_THREADS=str(cores),
+               MKL_NUM_THREADS=str(cores), CUDA_VISIBLE_DEVICES="")
+    code = (f"import json,sys; sys.path.insert(0,{ROOT!r}); import bench; "
+            f"print(json.dumps(bench.oracle_sample({workload!r}, {tokens}, {repeats})))")
+    r = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True,
+                       timeout=900)
+    if r.returncode:
+        raise RuntimeError(r.stderr[-2000:])
+    res = json.loads(r.stdout.strip().splitlines()[-1])
+    res["cores"] = cores
+    return res
+
+
+def run_reference(a):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    sh = mi.shape_by_name(a.workload)
+    # per-step sample sized from one probe step so that the whole run stays ~3 minutes
+    probe = cpu_baseline(a.workload, 64, 1)
+    per_tok = probe["seconds"][0] / 64
+    budget = 180.0 / max(1, a.steps + a.warmup)
+    tokens = int(max(sh.n_parties, min(sh.T, budget / max(per_tok, 1e-9))))
+    res = cpu_baseline(a.workload, tokens, a.steps + a.warmup)
+    secs = res["seconds"][a.warmup:]
+    ms = 1e3 * statistics.mean(secs)
+    value = res["tokens"] / (ms / 1e3)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
+        "n_gpus": a.gpus, "steps": a.steps, "warmup": a.warmup, "ms_per_step": ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (seeded numpy PCG64)",
+        "config": {"workload": workload_desc(sh), "sample_tokens": res["tokens"]},
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": res["cores"],
+                         "kind": "oracle",
+                         "sample": f"first {res['tokens']} tokens of {sh.name}, all experts, "
+                                   f"fp64 fwd+bwd per step"},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
+
+
+# --------------------------------------------------------------------------- our arm
+def main():
+    a = args_()
+    if a.impl == "reference":
+        run_reference(a)
+        return
+    import torch
+    import torch.distributed as dist
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    from paper_2506_02965_gb300.layer import MoELayer
+    sh = mi.shape_by_name(a.workload)
+    inp = mi.make_inputs(sh)
+    lay = MoELayer(sh)
+    lay.load(inp)
+    flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+    stream = torch.cuda.current_stream()
+
+    for i in range(max(3, a.warmup)):
+        flush.fill_(i & 0xFF)
+        lay.step()
+    torch.cuda.synchronize()
+    lay.check_status()
+
+    K = a.steps
+    names = ["start", "ffn_fwd_begin", "ffn_fwd_end", "ffn_bwd_begin", "ffn_bwd_end", "end"]
+    ev = [{n: torch.cuda.Event(enable_timing=True) for n in names} for _ in range(K)]
+    clocks = ClockSampler(local, enabled=not a.no_clocks)
+    time.sleep(0.3 if clocks.proc else 0)
+    barrier()
+    torch.cuda.synchronize()
+    t_wall = time.perf_counter()
+    for i in range(K):
+        flush.fill_(i & 0xFF)
+        e = ev[i]
+        e["start"].record(stream)
+        lay.step(mark=lambda n, e=e: e[n].record(stream))
+        e["end"].record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    wall = time.perf_counter() - t_wall
+    clk = clocks.stop()
+    lay.check_status()
+
+    step_ms = [e["start"].elapsed_time(e["end"]) for e in ev]
+    gemm_ms = [e["ffn_fwd_begin"].elapsed_time(e["ffn_fwd_end"]) +
+               e["ffn_bwd_begin"].elapsed_time(e["ffn_bwd_end"]) for e in ev]
+    ms = statistics.mean(step_ms)
+    gms = statistics.mean(gemm_ms)
+    if world > 1:
+        t = torch.tensor([ms, gms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms, gms = t.tolist()
+    value = world * sh.T / (ms / 1e3)
+
+    # e2e: host buffers in, host results out, through the same public calls
+    e2e = None
+    if not a.no_e2e:
+        hx = torch.from_numpy(inp["x"]).to(lay.dt).pin_memory()
+        hd = torch.from_numpy(inp["dout"]).to(lay.dt).pin_memory()
+        ho, hdx = torch.empty_like(hx).pin_memory(), torch.empty_like(hx).pin_memory()
+        hloss = torch.empty(sh.n_parties, dtype=torch.float32).pin_memory()
+        Ke = max(3, min(K, 100))
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        barrier()
+        torch.cuda.synchronize()
+        times = []
+        for i in range(Ke):
+            flush.fill_(i & 0xFF)
+            e0.record(stream)
+            lay.x.copy_(hx, non_blocking=True)
+            lay.dout.copy_(hd, non_blocking=True)
+            lay.step()
+            ho.copy_(lay.out, non_blocking=True)
+            hdx.copy_(lay.dx, non_blocking=True)
+            hloss.copy_(lay.aux_loss, non_blocking=True)
+            e1.record(stream)
+            e1.synchronize()
+            times.append(e0.elapsed_time(e1))
+        ems = statistics.mean(times)
+        if world > 1:
+            t = torch.tensor([ems], device="cuda")
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            ems = t.item()
+        nb = 2 if sh.dtype == "bf16" else 4
+        e2e = {"value": world * sh.T / (ems / 1e3), "unit": "tokens/s",
+               "h2d_bytes_per_step": 2 * sh.T * sh.d_model * nb,
+               "d2h_bytes_per_step": 2 * sh.T * sh.d_model * nb + 4 * sh.n_parties,
+               "ms_per_step": ems}
+        lay.check_status()
+
+    if rank != 0:
+        if world > 1:
+            dist.destroy_process_group()
+        return
+    pk = peaks()
+    gemm_flops = sh.gemm_flops()
+    achieved = gemm_flops / (gms / 1e3) / 1e12
+    n_gemm = 6 + (6 if sh.n_shared else 0)
+    traffic = gemm_traffic_record(sh)
+    roofline = {"bound": "tensor", "kernel": "grouped_gemm_kernel (tcgen05, all expert GEMM launches)",
+                "achieved": achieved, "peak": pk["bf16_tflops"], "unit": "TFLOP/s",
+                "frac": achieved / pk["bf16_tflops"], "traffic": traffic,
+                "launches_per_step": n_gemm,
+                "peak_source": f"{pk['source']} bf16 burst"}
+    mem_ms = ms - gms
+    mem_gbs = mem_bytes_per_step(sh) / (mem_ms / 1e3) / 1e9
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": K,
+        "warmup": a.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": sh.dtype,
+        "data": "synthetic (seeded numpy PCG64, BASELINE shapes, random-init weights)",
+        "config": {"workload": workload_desc(sh), "global_batch": world * sh.T,
+                   "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+                   "l2": "flushed (256 MiB write) before every timed step"},
+        "roofline": roofline,
+        "roofline_mem": {"bound": "hbm", "stages": "route, dispatch, combine, their bwd",
+                         "achieved": mem_gbs, "peak": pk["hbm_gbs"], "unit": "GB/s",
+                         "frac": mem_gbs / pk["hbm_gbs"],
+                         "note": "algorithmic bytes / (step time - expert GEMM time)"},
+        "gemm_ms_per_step": gms,
+        "gpu_launches": K * lay.kernels_per_step(),
+        "wall_s_timed": wall,
+    }
+    if e2e:
+        line["e2e"] = e2e
+    if clk:
+        line["clocks"] = clk
+    if world == 1 and not a.no_cpu_baseline:
+        try:
+            cb = cpu_baseline(a.workload, min(1024, sh.T), 2)
+            v = cb["tokens"] / min(cb["seconds"])
+            line["cpu_baseline"] = {"value": v, "unit": "tokens/s", "cores": cb["cores"],
+                                    "kind": "oracle",
+                                    "sample": f"first {cb['tokens']} tokens of {sh.name}, all "
+                                              f"experts, fp64 fwd+bwd, best of 2"}
+        except Exception as ex:  # reported, not fatal
+            line["cpu_baseline"] = {"error": str(ex)[-300:]}
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,351 @@
+// Token dispatch (the "send h to the host of idx" step of Alg. 3 as one expert-major
+// buffer), the gate-weighted combine of Alg. 3 and the backward of both (Alg. 5,
+// Sec. 3.2). All memory-bound: 16-byte vector loads/stores, one warp per token or
+// per permuted row, no floating-point atomics (every result is deterministic).
+#include "moe_common.cuh"
+#include "moe_internal.h"
+
+namespace moe {
+
+constexpr int DCH = 128;  // tokens per dispatch chunk (one thread each)
+
+// Per chunk: how many of its (token, pick) pairs went to each expert. Also checks
+// that every index lies in [0, E) and that no token picks an expert twice.
+__global__ void __launch_bounds__(DCH) chunk_count_kernel(const int32_t* __restrict__ idx,
+                                                          int64_t T, int E, int k,
+                                                          int32_t* chunk_counts) {
+    __shared__ int s_cnt[64];
+    for (int i = threadIdx.x; i < E; i += blockDim.x) s_cnt[i] = 0;
+    __syncthreads();
+    const int64_t t = (int64_t)blockIdx.x * DCH + threadIdx.x;
+    if (t < T) {
+        for (int j = 0; j < k; ++j) {
+            const int e = idx[t * k + j];
+            bool ok = (e >= 0 && e < E);
+            for (int jj = 0; jj < j; ++jj) ok = ok && (idx[t * k + jj] != e);
+            if (ok) atomicAdd(&s_cnt[e], 1);
+            else record_status(MOE_ERR_DEVICE_CHECK);
+        }
+    }
+    __syncthreads();
+    for (int i = threadIdx.x; i < E; i += blockDim.x)
+        chunk_counts[(int64_t)blockIdx.x * E + i] = s_cnt[i];
+}
+
+// Per chunk: offsets (written by chunk 0), the chunk's base row inside each expert
+// segment, and the stable rank of each pick among the chunk's picks of that expert
+// (a bit per token and expert, counted with popc).
+__global__ void __launch_bounds__(DCH) slot_kernel(const int32_t* __restrict__ idx,
+                                                   const int32_t* __restrict__ chunk_counts,
+                                                   int64_t T, int E, int k, int nchunks,
+                                                   int32_t* offsets, int32_t* slot_of,
+                                                   int32_t* token_of) {
+    __shared__ int s_pre[64];
+    __shared__ int s_tot[64];
+    __shared__ int s_base[64];
+    __shared__ unsigned s_bits[64][DCH / 32];
+    const int c = blockIdx.x;
+    for (int e = threadIdx.x; e < E; e += blockDim.x) {
+        int pre = 0, tot = 0;
+        for (int cc = 0; cc < nchunks; ++cc) {
+            const int v = chunk_counts[(int64_t)cc * E + e];
+            if (cc < c) pre += v;
+            tot += v;
+        }
+        s_pre[e] = pre;
+        s_tot[e] = tot;
+    }
+    for (int i = threadIdx.x; i < 64 * (DCH / 32); i += blockDim.x) (&s_bits[0][0])[i] = 0u;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int run = 0;
+        for (int e = 0; e < E; ++e) {
+            if (c == 0) offsets[e] = run;
+            s_base[e] = run + s_pre[e];
+            run += s_tot[e];
+        }
+        if (c == 0) offsets[E] = run;
+    }
+    const int i = threadIdx.x;
+    const int64_t t = (int64_t)c * DCH + i;
+    int es[8];
+    int kk = 0;
+    if (t < T) {
+        for (int j = 0; j < k; ++j) {
+            const int e = idx[t * k + j];
+            bool ok = (e >= 0 && e < E);
+            for (int jj = 0; jj < j; ++jj) ok = ok && (es[jj] != e);
+            es[j] = ok ? e : -1;
+            if (ok) atomicOr(&s_bits[e][i >> 5], 1u << (i & 31));
+            else slot_of[t * k + j] = -1;
+        }
+        kk = k;
+    }
+    __syncthreads();
+    for (int j = 0; j < kk; ++j) {
+        const int e = es[j];
+        if (e < 0) continue;
+        int rank = 0;
+        for (int w = 0; w < (i >> 5); ++w) rank += __popc(s_bits[e][w]);
+        rank += __popc(s_bits[e][i >> 5] & ((1u << (i & 31)) - 1u));
+        const int slot = s_base[e] + rank;
+        slot_of[t * k + j] = slot;
+        token_of[slot] = (int32_t)t;
+    }
+}
+
+// x_perm[r] = x[token_of[r]]: one warp per permuted row, 16-byte vectors.
+template <typename T>
+__global__ void __launch_bounds__(256) gather_kernel(const T* __restrict__ x,
+                                                     const int32_t* __restrict__ token_of,
+                                                     int64_t TK, int64_t Tn, int d, T* x_perm) {
+    const int lane = threadIdx.x & 31;
+    const int64_t r = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    if (r >= TK) return;
+    const int64_t t = token_of[r];
+    if (t < 0 || t >= Tn) {
+        if (lane == 0) record_status(MOE_ERR_DEVICE_CHECK);
+        return;
+    }
+    constexpr int VN = Vec<T>::N;
+    const int nv = d / VN;
+    const T* src = x + t * d;
+    T* dst = x_perm + r * d;
+    for (int v = lane; v < nv; v += 32) Vec<T>::raw_store(dst + v * VN, Vec<T>::raw_load(src + v * VN));
+}
+
+// out[t] = sum_j w[t,j] * y_perm[slot_of[t,j]] (+ sum_s y_sh[s,t]); fp32 accumulation.
+template <typename T>
+__global__ void __launch_bounds__(256) combine_fwd_kernel(const T* __restrict__ y_perm,
+                                                          const float* __restrict__ w,
+                                                          const int32_t* __restrict__ slot_of,
+                                                          const T* __restrict__ y_sh, int S,
+                                                          int64_t Tn, int d, int k, T* out) {
+    const int lane = threadIdx.x & 31;
+    const int64_t t = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    if (t >= Tn) return;
+    constexpr int VN = Vec<T>::N;
+    int64_t slot[8];
+    float wt[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+        slot[j] = j < k ? slot_of[t * k + j] : 0;
+        wt[j] = j < k ? w[t * k + j] : 0.f;
+        if (slot[j] < 0 || slot[j] >= Tn * k) {  // bad table: contribute nothing
+            if (lane == 0) record_status(MOE_ERR_DEVICE_CHECK);
+            slot[j] = 0;
+            wt[j] = 0.f;
+        }
+    }
+    const int nv = d / VN;
+    for (int v = lane; v < nv; v += 32) {
+        float acc[VN];
+#pragma unroll
+        for (int q = 0; q < VN; ++q) acc[q] = 0.f;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            if (j < k) {
+                float yv[VN];
+                Vec<T>::load(y_perm + slot[j] * d + v * VN, yv);
+#pragma unroll
+                for (int q = 0; q < VN; ++q) acc[q] = fmaf(wt[j], yv[q], acc[q]);
+            }
+        }
+        for (int s = 0; s < S; ++s) {
+            float yv[VN];
+            Vec<T>::load(y_sh + ((int64_t)s * Tn + t) * d + v * VN, yv);
+#pragma unroll
+            for (int q = 0; q < VN; ++q) acc[q] += yv[q];
+        }
+        Vec<T>::store(out + t * d + v * VN, acc);
+    }
+}
+
+// dy_perm[slot(t,j)] = w[t,j] dout[t];  dw[t,j] = <dout[t], y_perm[slot(t,j)]>.
+template <typename T>
+__global__ void __launch_bounds__(256) combine_bwd_kernel(const T* __restrict__ dout,
+                                                          const T* __restrict__ y_perm,
+                                                          const float* __restrict__ w,
+                                                          const int32_t* __restrict__ slot_of,
+                                                          int64_t Tn, int d, int k, T* dy_perm,
+                                                          float* dw) {
+    const int lane = threadIdx.x & 31;
+    const int64_t t = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    if (t >= Tn) return;
+    constexpr int VN = Vec<T>::N;
+    int64_t slot[8];
+    float wt[8], part[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+        slot[j] = j < k ? slot_of[t * k + j] : 0;
+        wt[j] = j < k ? w[t * k + j] : 0.f;
+        part[j] = 0.f;
+        if (slot[j] < 0 || slot[j] >= Tn * k) {
+            if (lane == 0) record_status(MOE_ERR_DEVICE_CHECK);
+            slot[j] = -1;
+        }
+    }
+    const int nv = d / VN;
+    for (int v = lane; v < nv; v += 32) {
+        float g[VN];
+        Vec<T>::load(dout + t * d + v * VN, g);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            if (j < k && slot[j] >= 0) {
+                float yv[VN], dy[VN];
+                Vec<T>::load(y_perm + slot[j] * d + v * VN, yv);
+#pragma unroll
+                for (int q = 0; q < VN; ++q) {
+                    part[j] = fmaf(g[q], yv[q], part[j]);
+                    dy[q] = wt[j] * g[q];
+                }
+                Vec<T>::store(dy_perm + slot[j] * d + v * VN, dy);
+            }
+        }
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+        if (j < k) {
+            const float s = warp_sum(part[j]);
+            if (lane == 0) dw[t * k + j] = s;
+        }
+    }
+}
+
+// dx[t] = sum_j dx_perm[slot(t,j)] + sum_e dlogits[t,e] W_r[p(t)][e] + sum_s dx_sh[s,t].
+template <typename T>
+__global__ void __launch_bounds__(256) unpermute_reduce_kernel(
+    const T* __restrict__ dx_perm, const int32_t* __restrict__ slot_of,
+    const float* __restrict__ dz, const T* __restrict__ wr, const int32_t* __restrict__ po, int P,
+    const T* __restrict__ dx_sh, int S, int64_t Tn, int d, int E, int k, T* dx) {
+    __shared__ float s_dz[8][64];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int64_t t = (int64_t)blockIdx.x * (blockDim.x >> 5) + warp;
+    if (t >= Tn) return;
+    constexpr int VN = Vec<T>::N;
+    const int party = party_of(po, P, t);
+    if (lane < E) s_dz[warp][lane] = dz[t * E + lane];
+    if (lane + 32 < E) s_dz[warp][lane + 32] = dz[t * E + lane + 32];
+    __syncwarp();
+    int64_t slot[8];
+    bool ok[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+        slot[j] = j < k ? slot_of[t * k + j] : 0;
+        ok[j] = j < k && slot[j] >= 0 && slot[j] < Tn * k;
+        if (j < k && !ok[j] && lane == 0) record_status(MOE_ERR_DEVICE_CHECK);
+    }
+    const T* W = wr + (int64_t)party * E * d;
+    const int nv = d / VN;
+    for (int v = lane; v < nv; v += 32) {
+        float acc[VN];
+#pragma unroll
+        for (int q = 0; q < VN; ++q) acc[q] = 0.f;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            if (ok[j]) {
+                float g[VN];
+                Vec<T>::load(dx_perm + slot[j] * d + v * VN, g);
+#pragma unroll
+                for (int q = 0; q < VN; ++q) acc[q] += g[q];
+            }
+        }
+        for (int s = 0; s < S; ++s) {
+            float g[VN];
+            Vec<T>::load(dx_sh + ((int64_t)s * Tn + t) * d + v * VN, g);
+#pragma unroll
+            for (int q = 0; q < VN; ++q) acc[q] += g[q];
+        }
+        for (int e = 0; e < E; ++e) {
+            float wv[VN];
+            Vec<T>::load(W + (int64_t)e * d + v * VN, wv);
+            const float z = s_dz[warp][e];
+#pragma unroll
+            for (int q = 0; q < VN; ++q) acc[q] = fmaf(z, wv[q], acc[q]);
+        }
+        Vec<T>::store(dx + t * d + v * VN, acc);
+    }
+}
+
+// ----------------------------------------------------------------------------- launchers
+size_t dispatch_workspace(int64_t T, int E) {
+    const int64_t nch = (T + DCH - 1) / DCH;
+    return (size_t)nch * E * sizeof(int32_t) + 256;
+}
+
+cudaError_t launch_dispatch(const int32_t* topk_idx, const void* x, int64_t T, int d, int E, int k,
+                            bool bf16, int32_t* offsets, int32_t* slot_of, int32_t* token_of,
+                            void* x_perm, void* ws, cudaStream_t s) {
+    const int nch = (int)((T + DCH - 1) / DCH);
+    int32_t* cc = (int32_t*)ws;
+    if (T == 0) {
+        return cudaMemsetAsync(offsets, 0, sizeof(int32_t) * (E + 1), s);
+    }
+    chunk_count_kernel<<<nch, DCH, 0, s>>>(topk_idx, T, E, k, cc);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    slot_kernel<<<nch, DCH, 0, s>>>(topk_idx, cc, T, E, k, nch, offsets, slot_of, token_of);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    const int64_t TK = T * k;
+    const unsigned blocks = (unsigned)((TK + 7) / 8);
+    if (bf16)
+        gather_kernel<__nv_bfloat16><<<blocks, 256, 0, s>>>((const __nv_bfloat16*)x, token_of, TK, T,
+                                                            d, (__nv_bfloat16*)x_perm);
+    else
+        gather_kernel<float><<<blocks, 256, 0, s>>>((const float*)x, token_of, TK, T, d,
+                                                    (float*)x_perm);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_combine_fwd(const void* y_perm, const float* topk_w, const int32_t* slot_of,
+                               const void* y_sh, int S, int64_t T, int d, int k, bool bf16,
+                               void* out, cudaStream_t s) {
+    if (T == 0) return cudaSuccess;
+    const unsigned blocks = (unsigned)((T + 7) / 8);
+    if (bf16)
+        combine_fwd_kernel<__nv_bfloat16><<<blocks, 256, 0, s>>>(
+            (const __nv_bfloat16*)y_perm, topk_w, slot_of, (const __nv_bfloat16*)y_sh, S, T, d, k,
+            (__nv_bfloat16*)out);
+    else
+        combine_fwd_kernel<float><<<blocks, 256, 0, s>>>((const float*)y_perm, topk_w, slot_of,
+                                                         (const float*)y_sh, S, T, d, k, (float*)out);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_combine_bwd(const void* dout, const void* y_perm, const float* topk_w,
+                               const int32_t* slot_of, int64_t T, int d, int k, bool bf16,
+                               void* dy_perm, float* dtopk_w, cudaStream_t s) {
+    if (T == 0) return cudaSuccess;
+    const unsigned blocks = (unsigned)((T + 7) / 8);
+    if (bf16)
+        combine_bwd_kernel<__nv_bfloat16><<<blocks, 256, 0, s>>>(
+            (const __nv_bfloat16*)dout, (const __nv_bfloat16*)y_perm, topk_w, slot_of, T, d, k,
+            (__nv_bfloat16*)dy_perm, dtopk_w);
+    else
+        combine_bwd_kernel<float><<<blocks, 256, 0, s>>>((const float*)dout, (const float*)y_perm,
+                                                         topk_w, slot_of, T, d, k, (float*)dy_perm,
+                                                         dtopk_w);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_unpermute_reduce(const void* dx_perm, const int32_t* slot_of,
+                                    const float* dlogits, const void* w_router,
+                                    const int32_t* po, int P, const void* dx_sh, int S, int64_t T,
+                                    int d, int E, int k, bool bf16, void* dx, cudaStream_t s) {
+    if (T == 0) return cudaSuccess;
+    const unsigned blocks = (unsigned)((T + 7) / 8);
+    if (bf16)
+        unpermute_reduce_kernel<__nv_bfloat16><<<blocks, 256, 0, s>>>(
+            (const __nv_bfloat16*)dx_perm, slot_of, dlogits, (const __nv_bfloat16*)w_router, po, P,
+            (const __nv_bfloat16*)dx_sh, S, T, d, E, k, (__nv_bfloat16*)dx);
+    else
+        unpermute_reduce_kernel<float><<<blocks, 256, 0, s>>>(
+            (const float*)dx_perm, slot_of, dlogits, (const float*)w_router, po, P,
+            (const float*)dx_sh, S, T, d, E, k, (float*)dx);
+    return cudaGetLastError();
+}
+
+cudaError_t dispatch_status(cudaStream_t s, int* code) { return tu_status_read_clear(s, code); }
+
+}  // namespace moe

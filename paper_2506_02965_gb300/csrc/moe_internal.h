@@ -1,0 +1,125 @@
+// Launchers shared between the kernel translation units and the C ABI (host side).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+namespace moe {
+
+struct RouteArgs {
+    const void* x;          // [T,d] dtype
+    const void* w_router;   // [P,E,d] dtype
+    const float* bias;      // [P,E] or null
+    const float* logits_in; // [T,E] (from-logits path)
+    const int32_t* po;      // [P+1] or null
+    int P;
+    int64_t T;
+    int d, E, k, normalize;
+    float* logits;
+    float* probs;
+    int32_t* topk_idx;
+    float* topk_w;
+    int32_t* counts;        // [P,E]
+};
+
+struct RouteBwdArgs {
+    const void* x;
+    const float* probs;
+    const int32_t* topk_idx;
+    const float* topk_w;
+    const float* dtopk_w;
+    const float* aux_coef;  // [P,E] or null
+    const int32_t* po;
+    int P;
+    int64_t T;
+    int d, E, k, normalize;
+    float* dlogits;
+    void* dw_router;
+    float* dbias;
+};
+
+cudaError_t launch_route(const RouteArgs& a, bool bf16, bool from_logits, cudaStream_t s);
+cudaError_t launch_aux_loss(const float* probs, const int32_t* counts, const int32_t* po, int P,
+                            int64_t T, int E, int k, float alpha, float* loss, float* coef,
+                            cudaStream_t s);
+size_t route_bwd_workspace(int64_t T, int P, int E, int d);
+cudaError_t launch_route_bwd(const RouteBwdArgs& a, bool bf16, void* ws, cudaStream_t s);
+cudaError_t route_status(cudaStream_t s, int* code);
+
+// dispatch / combine
+size_t dispatch_workspace(int64_t T, int E);
+cudaError_t launch_dispatch(const int32_t* topk_idx, const void* x, int64_t T, int d, int E, int k,
+                            bool bf16, int32_t* offsets, int32_t* slot_of, int32_t* token_of,
+                            void* x_perm, void* ws, cudaStream_t s);
+cudaError_t launch_combine_fwd(const void* y_perm, const float* topk_w, const int32_t* slot_of,
+                               const void* y_sh, int S, int64_t T, int d, int k, bool bf16,
+                               void* out, cudaStream_t s);
+cudaError_t launch_combine_bwd(const void* dout, const void* y_perm, const float* topk_w,
+                               const int32_t* slot_of, int64_t T, int d, int k, bool bf16,
+                               void* dy_perm, float* dtopk_w, cudaStream_t s);
+cudaError_t launch_unpermute_reduce(const void* dx_perm, const int32_t* slot_of,
+                                    const float* dlogits, const void* w_router,
+                                    const int32_t* po, int P, const void* dx_sh, int S, int64_t T,
+                                    int d, int E, int k, bool bf16, void* dx, cudaStream_t s);
+cudaError_t dispatch_status(cudaStream_t s, int* code);
+
+// grouped GEMMs -------------------------------------------------------------------------
+enum EpiKind { EPI_SWIGLU_FWD = 0, EPI_STORE = 1, EPI_SWIGLU_BWD = 2 };
+
+// How the groups (experts) of a grouped GEMM are laid out along the rows that vary:
+//  OFFSETS: group g owns rows [offsets[g], offsets[g+1]) of A / out (M-variable) or of
+//           both operands (K-variable);
+//  UNIFORM: every group has `rows` rows; group g starts at g*a_stride in A (or in the
+//           first operand), g*b_stride in the second operand (K-variable) and at
+//           g*out_stride in the output.
+struct GroupRows {
+    const int32_t* offsets;  // OFFSETS mode when non-null
+    int rows;                // UNIFORM: rows per group; OFFSETS: total rows of all groups
+    int64_t a_stride, b_stride, out_stride;
+};
+
+// C[M_g, N] = A_g[M_g, K] * B_g[N, K]^T per group g, M varying per group.
+//  A: [rows, K] dtype row-major (rows of all groups)
+//  B: group g's weight at b + g * b_group_elems, viewed as [N, K] (b_kmajor) or as
+//     [K, N] (MN-major, i.e. the transpose is stored)
+struct GemmMArgs {
+    int G;                 // groups
+    GroupRows rows;
+    const void* a;
+    const void* b;
+    int64_t b_group_elems;
+    bool b_kmajor;
+    int N, K;
+    int epi;
+    // EPI_SWIGLU_FWD: out0 = h_gu [rows, 2F] (G at cols [0,F), U at [F,2F)),
+    //                 out1 = act [rows, F]; N = 2F (B holds gate rows then up rows).
+    // EPI_STORE:      out0 = [rows, N].
+    // EPI_SWIGLU_BWD: aux = h_gu [rows, 2F] (input), out0 = dh [rows, 2F]; N = F.
+    void* out0;
+    void* out1;
+    const void* aux;
+};
+
+// C_g[M, N] = sum over the rows r of group g of A[r, m] * B[r, n]  (K varies per group)
+//  A: [rows, M] row-major; B: [rows, N] row-major; C: out + g*M*N, [M, N] row-major.
+struct GemmKArgs {
+    int G;
+    GroupRows rows;
+    const void* a;
+    const void* b;
+    int M, N;
+    void* out;
+};
+
+cudaError_t launch_gemm_m(const GemmMArgs& g, bool bf16, cudaStream_t s);
+cudaError_t launch_gemm_k(const GemmKArgs& g, bool bf16, cudaStream_t s);
+void set_wait_limit_ns(uint64_t ns);
+cudaError_t gemm_status(cudaStream_t s, int* code);
+cudaError_t simt_status(cudaStream_t s, int* code);
+
+// fp32 SIMT versions (the fp32 configuration); same argument meaning.
+cudaError_t launch_gemm_m_simt(const GemmMArgs& g, cudaStream_t s);
+cudaError_t launch_gemm_k_simt(const GemmKArgs& g, cudaStream_t s);
+
+}  // namespace moe

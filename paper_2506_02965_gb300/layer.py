@@ -1,0 +1,151 @@
+"""One MoE expert layer on the GPU: buffers in HBM and the fwd+bwd call sequence.
+
+torch provides device memory and streams only; every step runs in the CUDA
+library through the C ABI (``_lib``). The sequence is the layer's hot path:
+
+  forward : moe_route -> moe_aux_loss -> moe_dispatch -> moe_expert_ffn_fwd -> moe_combine_fwd
+  backward: moe_combine_bwd -> moe_expert_ffn_bwd -> moe_route_bwd -> moe_dispatch_bwd
+
+Layouts (row-major): x, out, dout, dx [T,d]; w_router [P,E,d]; w1 [E,2F,d] (gate
+rows then up rows); w2 [E,d,F]; x_perm, y_perm, dy_perm, dx_perm [T*k,d];
+h_gu, dh [T*k,2F]; act [T*k,F]; shared experts [S,...] likewise.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+from . import _lib as L
+
+
+class MoELayer:
+    def __init__(self, shape, device: str = "cuda"):
+        self.shape = sh = shape
+        self.device = device
+        self.dt = torch.bfloat16 if sh.dtype == "bf16" else torch.float32
+        self.cfg = L.make_config(sh.T, sh.d_model, sh.n_experts, sh.d_ff, sh.top_k, sh.n_parties,
+                                 sh.n_shared, sh.d_ff_shared, sh.normalize_topk, sh.aux_alpha,
+                                 L.MOE_BF16 if sh.dtype == "bf16" else L.MOE_F32)
+        T, d, E, F, k, P = sh.T, sh.d_model, sh.n_experts, sh.d_ff, sh.top_k, sh.n_parties
+        S, Fs, TK = sh.n_shared, sh.d_ff_shared, sh.T * sh.top_k
+        dt, f32, i32 = self.dt, torch.float32, torch.int32
+
+        def z(*s, dtype=dt):
+            return torch.empty(*s, dtype=dtype, device=device)
+
+        # parameters and inputs
+        self.x, self.dout = z(T, d), z(T, d)
+        self.w_router = z(P, E, d)
+        self.router_bias = None
+        self.party_offsets = z(P + 1, dtype=i32)
+        self.w1, self.w2 = z(E, 2 * F, d), z(E, d, F)
+        self.ws1 = z(S, 2 * Fs, d) if S else None
+        self.ws2 = z(S, d, Fs) if S else None
+        # forward
+        self.logits, self.probs = z(T, E, dtype=f32), z(T, E, dtype=f32)
+        self.topk_idx, self.topk_w = z(T, k, dtype=i32), z(T, k, dtype=f32)
+        self.counts = z(P, E, dtype=i32)
+        self.aux_loss, self.aux_coef = z(P, dtype=f32), z(P, E, dtype=f32)
+        self.offsets = z(E + 1, dtype=i32)
+        self.slot_of, self.token_of = z(TK, dtype=i32), z(TK, dtype=i32)
+        self.x_perm = z(TK, d)
+        self.h_gu, self.act, self.y_perm = z(TK, 2 * F), z(TK, F), z(TK, d)
+        self.h_gu_sh = z(S, T, 2 * Fs) if S else None
+        self.act_sh = z(S, T, Fs) if S else None
+        self.y_sh = z(S, T, d) if S else None
+        self.out = z(T, d)
+        # backward
+        self.dy_perm, self.dtopk_w = z(TK, d), z(T, k, dtype=f32)
+        self.dh, self.dx_perm = z(TK, 2 * F), z(TK, d)
+        self.dw1, self.dw2 = z(E, 2 * F, d), z(E, d, F)
+        self.dh_sh = z(S, T, 2 * Fs) if S else None
+        self.dx_sh = z(S, T, d) if S else None
+        self.dws1 = z(S, 2 * Fs, d) if S else None
+        self.dws2 = z(S, d, Fs) if S else None
+        self.dlogits = z(T, E, dtype=f32)
+        self.dw_router = z(P, E, d)
+        self.dbias = z(P, E, dtype=f32)
+        self.dx = z(T, d)
+        self.ws_bytes = L.moe_workspace_size(self.cfg)
+        self.workspace = torch.empty(max(self.ws_bytes, 16), dtype=torch.uint8, device=device)
+
+    # ------------------------------------------------------------------ inputs
+    def load(self, inp: dict):
+        """Copy seeded numpy inputs (synth.make_inputs) into the device buffers."""
+        def put(dst, a):
+            dst.copy_(torch.from_numpy(np.ascontiguousarray(a)).to(dst.dtype))
+
+        put(self.x, inp["x"])
+        put(self.dout, inp["dout"])
+        put(self.w_router, inp["w_router"])
+        put(self.party_offsets, inp["party_offsets"].astype(np.int32))
+        if inp.get("router_bias") is not None:
+            self.router_bias = torch.empty(self.shape.n_parties, self.shape.n_experts,
+                                           dtype=torch.float32, device=self.device)
+            put(self.router_bias, inp["router_bias"])
+        if "w1" in inp:
+            put(self.w1, inp["w1"])
+            put(self.w2, inp["w2"])
+            if self.shape.n_shared:
+                put(self.ws1, inp["ws1"])
+                put(self.ws2, inp["ws2"])
+
+    def _po(self):
+        return self.party_offsets if self.shape.n_parties > 1 else None
+
+    # ------------------------------------------------------------------ passes
+    def forward(self, stream=None, mark=None):
+        c = self.cfg
+        mark = mark or (lambda name: None)
+        L.moe_route(c, self.x, self.w_router, self.router_bias, self._po(), self.logits,
+                    self.probs, self.topk_idx, self.topk_w, self.counts, stream=stream)
+        L.moe_aux_loss(c, self.probs, self.counts, self._po(), self.aux_loss, self.aux_coef,
+                       stream=stream)
+        L.moe_dispatch(c, self.topk_idx, self.x, self.offsets, self.slot_of, self.token_of,
+                       self.x_perm, self.workspace, self.ws_bytes, stream=stream)
+        mark("ffn_fwd_begin")
+        L.moe_expert_ffn_fwd(c, self.x_perm, self.offsets, self.w1, self.w2, self.h_gu, self.act,
+                             self.y_perm, self.x, self.ws1, self.ws2, self.h_gu_sh, self.act_sh,
+                             self.y_sh, stream=stream)
+        mark("ffn_fwd_end")
+        L.moe_combine_fwd(c, self.y_perm, self.topk_w, self.slot_of, self.y_sh, self.out,
+                          stream=stream)
+
+    def backward(self, stream=None, with_aux: bool = True, mark=None):
+        c = self.cfg
+        mark = mark or (lambda name: None)
+        L.moe_combine_bwd(c, self.dout, self.y_perm, self.topk_w, self.slot_of, self.dy_perm,
+                          self.dtopk_w, stream=stream)
+        mark("ffn_bwd_begin")
+        L.moe_expert_ffn_bwd(c, self.x_perm, self.offsets, self.w1, self.w2, self.h_gu, self.act,
+                             self.dy_perm, self.dh, self.dx_perm, self.dw1, self.dw2, self.x,
+                             self.dout, self.ws1, self.ws2, self.h_gu_sh, self.act_sh, self.dh_sh,
+                             self.dx_sh, self.dws1, self.dws2, stream=stream)
+        mark("ffn_bwd_end")
+        L.moe_route_bwd(c, self.x, self.w_router, self.probs, self.topk_idx, self.topk_w,
+                        self.dtopk_w, self.aux_coef if with_aux else None, self._po(),
+                        self.dlogits, self.dw_router, self.dbias, self.workspace, self.ws_bytes,
+                        stream=stream)
+        L.moe_dispatch_bwd(c, self.dx_perm, self.slot_of, self.dlogits, self.w_router, self._po(),
+                           self.dx_sh, self.dx, stream=stream)
+
+    def step(self, stream=None, mark=None):
+        """One fwd+bwd pass of the whole layer. ``mark(name)`` (optional) is called at
+        the boundaries of the expert-GEMM calls: ffn_fwd_begin/end, ffn_bwd_begin/end."""
+        self.forward(stream, mark=mark)
+        self.backward(stream, mark=mark)
+
+    def kernels_per_step(self) -> int:
+        """CUDA kernels this library launches per step (memsets not counted):
+        route 1, aux 1, dispatch 3, expert fwd 2, combine 1, combine bwd 1,
+        expert bwd 4, route bwd 2, unpermute-reduce 1; shared experts add 2 + 4."""
+        return 16 + (6 if self.shape.n_shared else 0)
+
+    def check_status(self, stream=None):
+        code = L.moe_device_status(stream)
+        if code:
+            raise L.MoEError(code, "device", L.moe_status_string(code))
+
+    # ------------------------------------------------------------------ accounting
+    def gemm_flops(self) -> float:
+        return self.shape.gemm_flops()

@@ -1,0 +1,109 @@
+"""Host-side checks of the C ABI library (no GPU needed).
+
+The library must load, export every entry point include/moe.h declares, agree with
+the binding on the config struct layout, and reject bad arguments on the host
+before any CUDA call. The product path must not import the oracle.
+"""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "moe.h")
+
+
+@pytest.fixture(scope="module")
+def L():
+    from paper_2506_02965_gb300 import build as b
+    if not os.path.exists(b.LIB) or b._stale(b.LIB, os.path.join(b.CSRC, "moe_abi.cu")):
+        b.build()
+    from paper_2506_02965_gb300 import _lib
+    return _lib
+
+
+def declared_symbols():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(moe_[a-z_]+)\s*\(", text)))
+
+
+def test_every_declared_symbol_is_exported(L):
+    syms = declared_symbols()
+    assert len(syms) >= 16
+    for s in syms:
+        assert hasattr(L._lib, s), s
+        assert s in L.EXPORTED, s
+
+
+def test_config_struct_layout(L):
+    c = L.moe_config
+    assert ctypes.sizeof(c) == 48
+    names = [f[0] for f in c._fields_]
+    hdr = open(HEADER).read()
+    body = hdr[hdr.index("typedef struct {\n    int64_t T;"):hdr.index("} moe_config;")]
+    order = re.findall(r"\b(T|d_model|n_experts|d_ff|top_k|n_parties|n_shared|d_ff_shared|"
+                       r"normalize_topk|aux_alpha|dtype)\b", body)
+    assert order == names
+
+
+def test_status_strings_and_version(L):
+    assert L.moe_status_string(0) == "MOE_OK"
+    assert L.moe_status_string(4) == "MOE_ERR_TIMEOUT"
+    assert "sm_103a" in L.moe_version()
+
+
+def test_workspace_size_is_host_only(L):
+    cfg = L.make_config(4096, 1024, 16, 2816, 2)
+    n = L.moe_workspace_size(cfg)
+    assert n >= 4096 // 128 * 16 * 4
+
+
+@pytest.mark.parametrize("field,value,frag", [
+    ("n_experts", 0, "n_experts"), ("n_experts", 65, "n_experts"), ("top_k", 0, "top_k"),
+    ("top_k", 9, "top_k"), ("d_model", 100, "multiples of 128"), ("dtype", 7, "dtype"),
+    ("n_parties", 0, "n_parties"), ("normalize_topk", 2, "normalize_topk"), ("T", -1, "T="),
+])
+def test_bad_config_rejected_on_host(L, field, value, frag):
+    cfg = L.make_config(256, 256, 8, 256, 2)
+    setattr(cfg, field, value)
+    with pytest.raises(L.MoEError) as ei:
+        L.moe_route(cfg, 16, 16, None, None, 16, 16, 16, 16, 16, stream=0)
+    assert ei.value.status == L.MOE_ERR_INVALID_ARG
+    assert frag in L.moe_last_error()
+
+
+def test_null_and_misaligned_pointers_rejected_on_host(L):
+    cfg = L.make_config(256, 256, 8, 256, 2)
+    with pytest.raises(L.MoEError) as ei:
+        L.moe_route(cfg, None, 16, None, None, 16, 16, 16, 16, 16, stream=0)
+    assert ei.value.status == L.MOE_ERR_INVALID_ARG and "x is NULL" in L.moe_last_error()
+    with pytest.raises(L.MoEError):
+        L.moe_route(cfg, 18, 16, None, None, 16, 16, 16, 16, 16, stream=0)
+    assert "16-byte aligned" in L.moe_last_error()
+    cfg2 = L.make_config(256, 256, 8, 256, 2, n_parties=2)
+    with pytest.raises(L.MoEError):
+        L.moe_route(cfg2, 16, 16, None, None, 16, 16, 16, 16, 16, stream=0)
+    assert "party_offsets" in L.moe_last_error()
+    with pytest.raises(L.MoEError):
+        L.moe_dispatch(cfg, 16, 16, 16, 16, 16, 16, 16, 8, stream=0)
+    assert "workspace" in L.moe_last_error()
+    with pytest.raises(L.MoEError):
+        L.moe_set_wait_limit_ns(0)
+
+
+def test_binding_refuses_to_load_without_library(L, monkeypatch):
+    monkeypatch.setattr(L, "LIB_PATH", "/nonexistent/libmoe.so")
+    with pytest.raises(ImportError):
+        L._load()
+
+
+def test_product_path_does_not_touch_the_oracle():
+    pkg = os.path.join(ROOT, "paper_2506_02965_gb300")
+    for dp, _, fs in os.walk(pkg):
+        for f in fs:
+            if f.endswith((".py", ".cu", ".cuh", ".h")):
+                src = open(os.path.join(dp, f)).read()
+                assert not re.search(r"^\s*(from|import)\s+oracle", src, re.M), f
+                assert "oracle/" not in src, f

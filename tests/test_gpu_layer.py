@@ -1,0 +1,168 @@
+"""The whole layer, fwd+bwd through the C ABI, against the fp64 oracle.
+
+Full comparisons for the tiny fp32 workload and the mid-size bf16 workload at their
+own sizes, and for reduced-T versions of the fine-grained, Zipf and party workloads;
+sampled comparisons (per token, per feature column) at the full sizes of those three.
+Seeds are chosen by the oracle so that every compared token's routing is decided
+beyond the fp32 logit tolerance (oracle.seeds)."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import moe_oracle as mo
+from oracle import seeds
+from paper_2506_02965_gb300.layer import MoELayer
+from synth import moe_inputs as mi
+from tests._cmp import TOL, assert_close, ints, np64
+from tests.gpu_util import need_gpu, status
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def L():
+    return need_gpu()
+
+
+def run_layer(sh, inp):
+    lay = MoELayer(sh)
+    lay.load(inp)
+    lay.step()
+    torch.cuda.synchronize()
+    return lay
+
+
+def full_compare(lay, inp, sh):
+    tol = TOL[sh.dtype]
+    fwd = mo.layer_forward(inp, sh)
+    bwd = mo.layer_backward(inp, sh, fwd)
+    assert np.abs(np64(lay.logits) - fwd["logits"]).max() <= seeds.logit_tol(sh.d_model)
+    # integer work: bit-exact
+    assert (ints(lay.topk_idx) == fwd["topk_idx"]).all()
+    assert (ints(lay.counts) == fwd["party_counts"]).all()
+    assert (ints(lay.offsets) == fwd["offsets"]).all()
+    assert (ints(lay.slot_of) == fwd["slot_of"].ravel()).all()
+    assert (ints(lay.token_of) == fwd["token_of"]).all()
+    assert (np64(lay.x_perm) == fwd["x_perm"]).all()
+    errs = {}
+    for name, gpu, ref in [
+        ("probs", lay.probs, fwd["probs"]), ("topk_w", lay.topk_w, fwd["topk_w"]),
+        ("h_gu", lay.h_gu, fwd["h_gu"]), ("act", lay.act, fwd["act"]),
+        ("y_perm", lay.y_perm, fwd["y_perm"]), ("out", lay.out, fwd["out"]),
+        ("aux_loss", lay.aux_loss, fwd["aux_loss"]), ("aux_coef", lay.aux_coef, fwd["aux_coef"]),
+        ("dy_perm", lay.dy_perm, bwd["dy_perm"]), ("dtopk_w", lay.dtopk_w, bwd["dtopk_w"]),
+        ("dh", lay.dh, bwd["dh"]), ("dx_perm", lay.dx_perm, bwd["dx_perm"]),
+        ("dw1", lay.dw1, bwd["dw1"]), ("dw2", lay.dw2, bwd["dw2"]),
+        ("dlogits", lay.dlogits, bwd["dlogits"]), ("dw_router", lay.dw_router, bwd["dw_router"]),
+        ("dbias", lay.dbias, bwd["dbias"]), ("dx", lay.dx, bwd["dx"]),
+    ]:
+        errs[name] = assert_close(name, gpu, ref, tol)
+    for s in range(sh.n_shared):
+        G, U, A, Y = fwd["shared"][s]
+        dH, dX, dW1, dW2 = bwd["shared_grads"][s]
+        errs[f"y_sh{s}"] = assert_close("y_sh", lay.y_sh[s], Y, tol)
+        errs[f"dws1_{s}"] = assert_close("dws1", lay.dws1[s], dW1, tol)
+        errs[f"dws2_{s}"] = assert_close("dws2", lay.dws2[s], dW2, tol)
+    return errs
+
+
+SMALL = {
+    "tiny_f32": lambda: mi.SHAPES[1],
+    "tiny_f32_renorm": lambda: mi.SHAPES[1].with_(normalize_topk=1, aux_alpha=1.0),
+    "mid_bf16": lambda: mi.SHAPES[2],
+    "mid_bf16_renorm": lambda: mi.SHAPES[2].with_(T=1000, normalize_topk=1),
+    "fine_bf16_T512": lambda: mi.SHAPES[3].with_(T=512),
+    "large_zipf_bf16_T384": lambda: mi.SHAPES[4].with_(T=384),
+    "party4_bf16_T1024": lambda: mi.SHAPES[5].with_(T=1024),
+    "all_experts_k_eq_E": lambda: mi.MoEShape("kE", 200, 256, 4, 256, 4, "bf16", seed=77),
+    "one_token": lambda: mi.MoEShape("t1", 1, 128, 8, 128, 2, "bf16", seed=78),
+}
+
+
+@pytest.mark.parametrize("name", list(SMALL))
+def test_layer_full_parity(L, name):
+    sh = SMALL[name]()
+    sh = sh.with_(seed=seeds.decided_seed(sh))
+    inp = mi.make_inputs(sh)
+    lay = run_layer(sh, inp)
+    assert status(L) == 0
+    errs = full_compare(lay, inp, sh)
+    print(name, {k: f"{v:.2e}" for k, v in errs.items()})
+
+
+def test_layer_is_deterministic(L):
+    sh = mi.SHAPES[2].with_(T=1024)
+    inp = mi.make_inputs(sh)
+    a = run_layer(sh, inp)
+    b = run_layer(sh, inp)
+    for n in ("out", "dx", "dw1", "dw2", "dw_router", "dlogits", "dtopk_w", "slot_of"):
+        assert torch.equal(getattr(a, n), getattr(b, n)), n
+
+
+def test_layer_empty_batch(L):
+    sh = mi.MoEShape("empty", 0, 256, 8, 256, 2, "bf16")
+    lay = MoELayer(sh)
+    inp = mi.make_inputs(sh.with_(T=0))
+    lay.load(inp)
+    lay.dw1.fill_(1)
+    lay.step()
+    assert status(L) == 0
+    assert (ints(lay.offsets) == 0).all()
+    assert (lay.dw1 == 0).all() and (lay.dw2 == 0).all() and (lay.dw_router == 0).all()
+
+
+@pytest.mark.parametrize("which", [3, 4, 5])
+def test_layer_sampled_parity_full_size(L, which):
+    """Full-size workloads: every token's routing, sampled tokens' outputs and input
+    gradients, sampled weight-gradient slices, and dW_r against dlogits^T x."""
+    sh = mi.SHAPES[which]
+    inp = mi.make_inputs(sh)
+    lay = run_layer(sh, inp)
+    assert status(L) == 0
+    tol = TOL[sh.dtype]
+    route = mo.route_all(inp, sh)
+    z = route["logits"]
+    lt = seeds.logit_tol(sh.d_model)
+    assert np.abs(np64(lay.logits) - z).max() <= lt
+    margin = mo.top_margin(z, sh.top_k)
+    decided = margin > 2 * lt
+    idx = ints(lay.topk_idx)
+    assert (idx[decided] == route["topk_idx"][decided]).all()
+    # undecided tokens: the GPU picks must still be a valid top-k under its own logits
+    gl = np64(lay.logits)
+    for t in np.nonzero(~decided)[0]:
+        kth = np.sort(gl[t])[::-1][sh.top_k - 1]
+        assert (gl[t][idx[t]] >= kth).all()
+    flipped = np.nonzero((idx != route["topk_idx"]).any(axis=1))[0]
+    touched = set(route["topk_idx"][flipped].ravel().tolist()) | set(idx[flipped].ravel().tolist())
+    rng = np.random.default_rng(sh.seed)
+    toks = rng.choice(np.nonzero(decided)[0], size=48, replace=False)
+    toks = np.concatenate([toks, [0, sh.T - 1]]) if decided[0] and decided[-1] else toks
+    rows = mo.sampled_token_rows(inp, sh, route, toks)
+    toks_d = torch.as_tensor(toks, device="cuda")
+    # per-token rows are compared against the scale of the sampled reference
+    assert_close("out", lay.out[toks_d], rows["out"], tol)
+    assert_close("dx", lay.dx[toks_d], rows["dx"], tol)
+    assert_close("dtopk_w", lay.dtopk_w[toks_d], rows["dtopk_w"], tol)
+    assert_close("dlogits", lay.dlogits[toks_d], rows["dlogits"], tol)
+    slot = ints(lay.slot_of).reshape(sh.T, sh.top_k)
+    for i, t in enumerate(toks):
+        assert_close("y", lay.y_perm[torch.as_tensor(slot[t], device="cuda")], rows["y"][i], tol)
+    # weight-gradient slices of experts whose rows no flipped token touched
+    F = sh.d_ff
+    cols = sorted(rng.choice(F, size=4, replace=False).tolist())
+    experts = [e for e in rng.permutation(sh.n_experts)[:6] if e not in touched]
+    for e in experts:
+        sw = mo.sampled_weight_grads(inp, sh, route, int(e), cols)
+        assert_close("dw2 cols", lay.dw2[e][:, cols], sw["dw2_cols"], tol)
+        assert_close("dw1 gate rows", lay.dw1[e][cols], sw["dw1_gate_rows"], tol)
+        assert_close("dw1 up rows", lay.dw1[e][[F + c for c in cols]], sw["dw1_up_rows"], tol)
+    # router weight gradient: the GPU's dW_r equals dlogits^T x of its own dlogits
+    po = inp["party_offsets"]
+    dz = np64(lay.dlogits)
+    for p in range(sh.n_parties):
+        r = slice(po[p], po[p + 1])
+        ref = dz[r].T @ inp["x"][r].astype(np.float64)
+        assert_close("dw_router", lay.dw_router[p], ref, tol)
+        assert_close("dbias", lay.dbias[p], dz[r].sum(0), 1e-4)
+    assert (ints(lay.counts).sum() == sh.T * sh.top_k)
