@@ -125,6 +125,27 @@ moe_status moe_dispatch(const moe_config* cfg, const int32_t* topk_idx, const vo
                         void* workspace, size_t workspace_bytes, moe_stream_t stream);
 
 /*
+ * moe_dispatch without a workspace argument, for callers that cannot allocate device
+ * memory: code whose host framework hands it only input and output buffers (an op or
+ * plugin interface with no scratch), or that must not allocate while it runs (a
+ * fixed device-memory budget). The paper has no counterpart; this is a library
+ * convenience. Same arguments and results as moe_dispatch.
+ *  - Scratch: a fixed device array inside the library of 65536 int32 entries
+ *    (256 KiB), held by every GPU that loads the library until the process exits.
+ *    It bounds the size: ceil(T/128) * E <= 65536 (e.g. T <= 131072 with E = 64);
+ *    larger requests return MOE_ERR_INVALID_ARG and queue no work.
+ *  - Calls no cudaMalloc or cudaFree. The first call on a device looks up the
+ *    array's device address once (cudaGetSymbolAddress); make that first call before
+ *    any stream capture.
+ *  - Every call shares the one array. Each call overwrites the entries it uses, so
+ *    back-to-back calls on one stream are fine; calls whose kernels overlap on the GPU
+ *    (several streams or host threads at once) race and give wrong tables.
+ */
+moe_status moe_dispatch_noalloc(const moe_config* cfg, const int32_t* topk_idx, const void* x,
+                                int32_t* offsets, int32_t* slot_of, int32_t* token_of,
+                                void* x_perm, moe_stream_t stream);
+
+/*
  * ForwardExpert of Alg. 6 for every routed expert, on its rows of x_perm, plus the
  * always-on shared experts on every token. Expert e is SwiGLU:
  *   [G|U] = x_perm_e W1[e]^T, A = silu(G) * U, Y = A W2[e]^T

@@ -65,6 +65,7 @@ _SIGS = {
     "moe_route_from_logits": [_CFG] + [P] * 7,
     "moe_aux_loss": [_CFG] + [P] * 6,
     "moe_dispatch": [_CFG] + [P] * 7 + [ctypes.c_size_t, P],
+    "moe_dispatch_noalloc": [_CFG] + [P] * 7,
     "moe_expert_ffn_fwd": [_CFG] + [P] * 14,
     "moe_combine_fwd": [_CFG] + [P] * 6,
     "moe_combine_bwd": [_CFG] + [P] * 7,
@@ -173,6 +174,11 @@ def moe_dispatch(cfg, topk_idx, x, offsets, slot_of, token_of, x_perm, workspace
                  workspace_bytes, stream=None):
     _call("moe_dispatch", cfg, topk_idx, x, offsets, slot_of, token_of, x_perm, workspace,
           int(workspace_bytes), stream=stream)
+
+
+def moe_dispatch_noalloc(cfg, topk_idx, x, offsets, slot_of, token_of, x_perm, stream=None):
+    _call("moe_dispatch_noalloc", cfg, topk_idx, x, offsets, slot_of, token_of, x_perm,
+          stream=stream)
 
 
 def moe_expert_ffn_fwd(cfg, x_perm, offsets, w1, w2, h_gu, act, y_perm, x=None, ws1=None,

@@ -346,6 +346,56 @@ cudaError_t launch_unpermute_reduce(const void* dx_perm, const int32_t* slot_of,
     return cudaGetLastError();
 }
 
+// ----------------------------------------------------------------------------- no-alloc dispatch
+// Dispatch for callers that cannot allocate device memory (their interface hands them
+// only input and output buffers). The per-chunk counts live in this file-scope array
+// instead of a caller workspace: every GPU that loads the library holds it until the
+// process exits, and every call shares it. chunk_count_kernel overwrites each entry it
+// uses, so nothing has to be cleared between calls; calls whose kernels overlap on the
+// GPU (different streams, or several host threads) race on it.
+static __device__ __align__(256) int32_t g_dispatch_scratch[kNoAllocScratchInts];
+
+namespace {
+constexpr int kMaxDevices = 64;
+int32_t* g_scratch_ptr[kMaxDevices] = {};
+}  // namespace
+
+int64_t dispatch_noalloc_max_chunk_entries() { return kNoAllocScratchInts; }
+
+cudaError_t launch_dispatch_noalloc(const int32_t* topk_idx, const void* x, int64_t T, int d, int E,
+                                    int k, bool bf16, int32_t* offsets, int32_t* slot_of,
+                                    int32_t* token_of, void* x_perm, cudaStream_t s) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    if (!g_scratch_ptr[dev]) {  // first call on this device: look the array up once
+        void* p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_dispatch_scratch);
+        if (e != cudaSuccess) return e;
+        g_scratch_ptr[dev] = static_cast<int32_t*>(p);
+    }
+    int32_t* cc = g_scratch_ptr[dev];
+    const int nch = (int)((T + DCH - 1) / DCH);
+    if ((int64_t)nch * E > kNoAllocScratchInts) return cudaErrorInvalidValue;
+    if (T == 0) return cudaMemsetAsync(offsets, 0, sizeof(int32_t) * (E + 1), s);
+    chunk_count_kernel<<<nch, DCH, 0, s>>>(topk_idx, T, E, k, cc);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    slot_kernel<<<nch, DCH, 0, s>>>(topk_idx, cc, T, E, k, nch, offsets, slot_of, token_of);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    const int64_t TK = T * k;
+    const unsigned blocks = (unsigned)((TK + 7) / 8);
+    if (bf16)
+        gather_kernel<__nv_bfloat16><<<blocks, 256, 0, s>>>((const __nv_bfloat16*)x, token_of, TK, T,
+                                                            d, (__nv_bfloat16*)x_perm);
+    else
+        gather_kernel<float><<<blocks, 256, 0, s>>>((const float*)x, token_of, TK, T, d,
+                                                    (float*)x_perm);
+    return cudaGetLastError();
+}
+
 cudaError_t dispatch_status(cudaStream_t s, int* code) { return tu_status_read_clear(s, code); }
 
 }  // namespace moe

@@ -226,6 +226,31 @@ moe_status moe_dispatch(const moe_config* cfg, const int32_t* topk_idx, const vo
                        "moe_dispatch");
 }
 
+moe_status moe_dispatch_noalloc(const moe_config* cfg, const int32_t* topk_idx, const void* x,
+                                int32_t* offsets, int32_t* slot_of, int32_t* token_of,
+                                void* x_perm, moe_stream_t stream) {
+    moe_status st = check_cfg(cfg);
+    if (st) return st;
+    REQUIRE(offsets);
+    const int64_t nch = (cfg->T + 127) / 128;
+    if (nch * cfg->n_experts > dispatch_noalloc_max_chunk_entries())
+        return fail(MOE_ERR_INVALID_ARG,
+                    "moe_dispatch_noalloc: ceil(T/128)*E = %lld exceeds its fixed scratch of %lld "
+                    "entries; use moe_dispatch with a workspace",
+                    (long long)(nch * cfg->n_experts), (long long)dispatch_noalloc_max_chunk_entries());
+    if (cfg->T > 0) {
+        REQUIRE(topk_idx);
+        REQUIRE_VEC(x);
+        REQUIRE(slot_of);
+        REQUIRE(token_of);
+        REQUIRE_VEC(x_perm);
+    }
+    return cuda_status(launch_dispatch_noalloc(topk_idx, x, cfg->T, cfg->d_model, cfg->n_experts,
+                                               cfg->top_k, cfg->dtype == MOE_BF16, offsets, slot_of,
+                                               token_of, x_perm, (cudaStream_t)stream),
+                       "moe_dispatch_noalloc");
+}
+
 moe_status moe_expert_ffn_fwd(const moe_config* cfg, const void* x_perm, const int32_t* offsets,
                               const void* w1, const void* w2, void* h_gu, void* act, void* y_perm,
                               const void* x, const void* ws1, const void* ws2, void* h_gu_sh,

@@ -63,6 +63,12 @@ cudaError_t launch_unpermute_reduce(const void* dx_perm, const int32_t* slot_of,
                                     const int32_t* po, int P, const void* dx_sh, int S, int64_t T,
                                     int d, int E, int k, bool bf16, void* dx, cudaStream_t s);
 cudaError_t dispatch_status(cudaStream_t s, int* code);
+// dispatch with its per-chunk counts in a fixed device array (no workspace argument)
+constexpr int64_t kNoAllocScratchInts = 1 << 16;  // 256 KiB of int32 chunk counts
+int64_t dispatch_noalloc_max_chunk_entries();
+cudaError_t launch_dispatch_noalloc(const int32_t* topk_idx, const void* x, int64_t T, int d, int E,
+                                    int k, bool bf16, int32_t* offsets, int32_t* slot_of,
+                                    int32_t* token_of, void* x_perm, cudaStream_t s);
 
 // grouped GEMMs -------------------------------------------------------------------------
 enum EpiKind { EPI_SWIGLU_FWD = 0, EPI_STORE = 1, EPI_SWIGLU_BWD = 2 };
