@@ -115,6 +115,10 @@ __global__ void __launch_bounds__(256) gather_kernel(const T* __restrict__ x,
 }
 
 // out[t] = sum_j w[t,j] * y_perm[slot_of[t,j]] (+ sum_s y_sh[s,t]); fp32 accumulation.
+// One warp per token; every lane issues the loads of up to UB vectors of all k rows
+// before it uses any of them, so enough bytes are in flight to keep HBM busy.
+constexpr int UB = 4;
+
 template <typename T>
 __global__ void __launch_bounds__(256) combine_fwd_kernel(const T* __restrict__ y_perm,
                                                           const float* __restrict__ w,
@@ -138,26 +142,39 @@ __global__ void __launch_bounds__(256) combine_fwd_kernel(const T* __restrict__ 
         }
     }
     const int nv = d / VN;
-    for (int v = lane; v < nv; v += 32) {
-        float acc[VN];
+    for (int v0 = lane; v0 < nv; v0 += 32 * UB) {
+        uint4 raw[UB][8];
 #pragma unroll
-        for (int q = 0; q < VN; ++q) acc[q] = 0.f;
+        for (int u = 0; u < UB; ++u) {
+            const int v = v0 + 32 * u;
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-            if (j < k) {
-                float yv[VN];
-                Vec<T>::load(y_perm + slot[j] * d + v * VN, yv);
+            for (int j = 0; j < 8; ++j)
+                if (j < k && v < nv) raw[u][j] = Vec<T>::raw_load(y_perm + slot[j] * d + v * VN);
+        }
 #pragma unroll
-                for (int q = 0; q < VN; ++q) acc[q] = fmaf(wt[j], yv[q], acc[q]);
+        for (int u = 0; u < UB; ++u) {
+            const int v = v0 + 32 * u;
+            if (v >= nv) break;
+            float acc[VN];
+#pragma unroll
+            for (int q = 0; q < VN; ++q) acc[q] = 0.f;
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                if (j < k) {
+                    float yv[VN];
+                    unpack_vec<T>(raw[u][j], yv);
+#pragma unroll
+                    for (int q = 0; q < VN; ++q) acc[q] = fmaf(wt[j], yv[q], acc[q]);
+                }
             }
-        }
-        for (int s = 0; s < S; ++s) {
-            float yv[VN];
-            Vec<T>::load(y_sh + ((int64_t)s * Tn + t) * d + v * VN, yv);
+            for (int s2 = 0; s2 < S; ++s2) {
+                float yv[VN];
+                Vec<T>::load(y_sh + ((int64_t)s2 * Tn + t) * d + v * VN, yv);
 #pragma unroll
-            for (int q = 0; q < VN; ++q) acc[q] += yv[q];
+                for (int q = 0; q < VN; ++q) acc[q] += yv[q];
+            }
+            Vec<T>::store(out + t * d + v * VN, acc);
         }
-        Vec<T>::store(out + t * d + v * VN, acc);
     }
 }
 
@@ -186,84 +203,146 @@ __global__ void __launch_bounds__(256) combine_bwd_kernel(const T* __restrict__ 
         }
     }
     const int nv = d / VN;
-    for (int v = lane; v < nv; v += 32) {
-        float g[VN];
-        Vec<T>::load(dout + t * d + v * VN, g);
+    for (int v0 = lane; v0 < nv; v0 += 32 * UB) {
+        uint4 graw[UB], yraw[UB][8];
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-            if (j < k && slot[j] >= 0) {
-                float yv[VN], dy[VN];
-                Vec<T>::load(y_perm + slot[j] * d + v * VN, yv);
+        for (int u = 0; u < UB; ++u) {
+            const int v = v0 + 32 * u;
+            if (v < nv) {
+                graw[u] = Vec<T>::raw_load(dout + t * d + v * VN);
 #pragma unroll
-                for (int q = 0; q < VN; ++q) {
-                    part[j] = fmaf(g[q], yv[q], part[j]);
-                    dy[q] = wt[j] * g[q];
+                for (int j = 0; j < 8; ++j)
+                    if (j < k && slot[j] >= 0) yraw[u][j] = Vec<T>::raw_load(y_perm + slot[j] * d + v * VN);
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < UB; ++u) {
+            const int v = v0 + 32 * u;
+            if (v >= nv) break;
+            float g[VN];
+            unpack_vec<T>(graw[u], g);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                if (j < k && slot[j] >= 0) {
+                    float yv[VN], dy[VN];
+                    unpack_vec<T>(yraw[u][j], yv);
+#pragma unroll
+                    for (int q = 0; q < VN; ++q) {
+                        part[j] = fmaf(g[q], yv[q], part[j]);
+                        dy[q] = wt[j] * g[q];
+                    }
+                    Vec<T>::store(dy_perm + slot[j] * d + v * VN, dy);
                 }
-                Vec<T>::store(dy_perm + slot[j] * d + v * VN, dy);
             }
         }
     }
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
         if (j < k) {
-            const float s = warp_sum(part[j]);
-            if (lane == 0) dw[t * k + j] = s;
+            const float sum = warp_sum(part[j]);
+            if (lane == 0) dw[t * k + j] = sum;
         }
     }
 }
 
 // dx[t] = sum_j dx_perm[slot(t,j)] + sum_e dlogits[t,e] W_r[p(t)][e] + sum_s dx_sh[s,t].
+// A block takes UR_TOK tokens of one party and a slab of 64 * VN columns: the party's
+// router rows for the slab and the tokens' dlogits are staged in shared memory; each
+// thread owns VN columns of UR_TOK / 4 tokens.
+constexpr int UR_TOK = 32;
+
 template <typename T>
 __global__ void __launch_bounds__(256) unpermute_reduce_kernel(
     const T* __restrict__ dx_perm, const int32_t* __restrict__ slot_of,
     const float* __restrict__ dz, const T* __restrict__ wr, const int32_t* __restrict__ po, int P,
     const T* __restrict__ dx_sh, int S, int64_t Tn, int d, int E, int k, T* dx) {
-    __shared__ float s_dz[8][64];
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int64_t t = (int64_t)blockIdx.x * (blockDim.x >> 5) + warp;
-    if (t >= Tn) return;
     constexpr int VN = Vec<T>::N;
-    const int party = party_of(po, P, t);
-    if (lane < E) s_dz[warp][lane] = dz[t * E + lane];
-    if (lane + 32 < E) s_dz[warp][lane + 32] = dz[t * E + lane + 32];
-    __syncwarp();
-    int64_t slot[8];
-    bool ok[8];
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-        slot[j] = j < k ? slot_of[t * k + j] : 0;
-        ok[j] = j < k && slot[j] >= 0 && slot[j] < Tn * k;
-        if (j < k && !ok[j] && lane == 0) record_status(MOE_ERR_DEVICE_CHECK);
+    constexpr int SLAB = 64 * VN;
+    constexpr int TPT = UR_TOK / 4;  // tokens per thread
+    extern __shared__ __align__(16) unsigned char ur_smem[];
+    float* s_dz = reinterpret_cast<float*>(ur_smem);                  // [UR_TOK][E]
+    T* s_w = reinterpret_cast<T*>(ur_smem + UR_TOK * 64 * sizeof(float));  // [E][SLAB]
+    // tile -> (party, first token)
+    int64_t ti = blockIdx.x, t0 = -1, tend = 0;
+    int party = 0;
+    for (int p = 0; p < P; ++p) {
+        const int64_t a = po ? po[p] : 0, b = po ? po[p + 1] : Tn;
+        const int64_t nt = (b - a + UR_TOK - 1) / UR_TOK;
+        if (ti < nt) { party = p; t0 = a + ti * UR_TOK; tend = b; break; }
+        ti -= nt;
     }
+    if (t0 < 0) return;
+    const int n = (int)min64(UR_TOK, tend - t0);
+    const int64_t c0 = (int64_t)blockIdx.y * SLAB;
+    const int ncols = (int)min64(SLAB, d - c0);
     const T* W = wr + (int64_t)party * E * d;
-    const int nv = d / VN;
-    for (int v = lane; v < nv; v += 32) {
-        float acc[VN];
+    for (int i = threadIdx.x; i < UR_TOK * E; i += blockDim.x) {
+        const int tt = i / E, e = i % E;
+        s_dz[i] = tt < n ? dz[(t0 + tt) * E + e] : 0.f;
+    }
+    for (int i = threadIdx.x; i < E * (SLAB / VN); i += blockDim.x) {
+        const int e = i / (SLAB / VN), v = i % (SLAB / VN);
+        if (v * VN < ncols) Vec<T>::raw_store(s_w + e * SLAB + v * VN, Vec<T>::raw_load(W + (int64_t)e * d + c0 + v * VN));
+    }
+    __syncthreads();
+    const int cv = threadIdx.x & 63;       // column vector inside the slab
+    const int tg = threadIdx.x >> 6;        // token group
+    if (cv * VN >= ncols) return;
+    float acc[TPT][VN];
 #pragma unroll
-        for (int q = 0; q < VN; ++q) acc[q] = 0.f;
+    for (int i = 0; i < TPT; ++i)
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-            if (ok[j]) {
-                float g[VN];
-                Vec<T>::load(dx_perm + slot[j] * d + v * VN, g);
+        for (int q = 0; q < VN; ++q) acc[i][q] = 0.f;
+    for (int e = 0; e < E; ++e) {
+        float wv[VN];
+        Vec<T>::load(s_w + e * SLAB + cv * VN, wv);
 #pragma unroll
-                for (int q = 0; q < VN; ++q) acc[q] += g[q];
+        for (int i = 0; i < TPT; ++i) {
+            const float zz = s_dz[(tg * TPT + i) * E + e];
+#pragma unroll
+            for (int q = 0; q < VN; ++q) acc[i][q] = fmaf(zz, wv[q], acc[i][q]);
+        }
+    }
+    const int64_t col = c0 + cv * VN;
+    // pick by pick: the slot lookups of this thread's tokens, then their rows, in flight
+    // together
+    for (int j = 0; j < k; ++j) {
+        int32_t slot[TPT];
+#pragma unroll
+        for (int i = 0; i < TPT; ++i) {
+            const int tt = tg * TPT + i;
+            slot[i] = tt < n ? slot_of[(t0 + tt) * k + j] : -1;
+            if (tt < n && (slot[i] < 0 || (int64_t)slot[i] >= Tn * k)) {
+                if (cv == 0) record_status(MOE_ERR_DEVICE_CHECK);
+                slot[i] = -1;
             }
         }
-        for (int s = 0; s < S; ++s) {
+        uint4 raw[TPT];
+#pragma unroll
+        for (int i = 0; i < TPT; ++i)
+            if (slot[i] >= 0) raw[i] = Vec<T>::raw_load(dx_perm + (int64_t)slot[i] * d + col);
+#pragma unroll
+        for (int i = 0; i < TPT; ++i) {
+            if (slot[i] >= 0) {
+                float g[VN];
+                unpack_vec<T>(raw[i], g);
+#pragma unroll
+                for (int q = 0; q < VN; ++q) acc[i][q] += g[q];
+            }
+        }
+    }
+#pragma unroll
+    for (int i = 0; i < TPT; ++i) {
+        const int tt = tg * TPT + i;
+        if (tt >= n) break;
+        const int64_t t = t0 + tt;
+        for (int s2 = 0; s2 < S; ++s2) {
             float g[VN];
-            Vec<T>::load(dx_sh + ((int64_t)s * Tn + t) * d + v * VN, g);
+            Vec<T>::load(dx_sh + ((int64_t)s2 * Tn + t) * d + col, g);
 #pragma unroll
-            for (int q = 0; q < VN; ++q) acc[q] += g[q];
+            for (int q = 0; q < VN; ++q) acc[i][q] += g[q];
         }
-        for (int e = 0; e < E; ++e) {
-            float wv[VN];
-            Vec<T>::load(W + (int64_t)e * d + v * VN, wv);
-            const float z = s_dz[warp][e];
-#pragma unroll
-            for (int q = 0; q < VN; ++q) acc[q] = fmaf(z, wv[q], acc[q]);
-        }
-        Vec<T>::store(dx + t * d + v * VN, acc);
+        Vec<T>::store(dx + t * d + col, acc[i]);
     }
 }
 
@@ -334,15 +413,36 @@ cudaError_t launch_unpermute_reduce(const void* dx_perm, const int32_t* slot_of,
                                     const int32_t* po, int P, const void* dx_sh, int S, int64_t T,
                                     int d, int E, int k, bool bf16, void* dx, cudaStream_t s) {
     if (T == 0) return cudaSuccess;
-    const unsigned blocks = (unsigned)((T + 7) / 8);
-    if (bf16)
-        unpermute_reduce_kernel<__nv_bfloat16><<<blocks, 256, 0, s>>>(
+    const unsigned tiles = (unsigned)((T + UR_TOK - 1) / UR_TOK + P);
+    const int VN = bf16 ? 8 : 4;
+    const int slab = 64 * VN;
+    dim3 grid(tiles, (d + slab - 1) / slab);
+    const size_t smem = UR_TOK * 64 * sizeof(float) + (size_t)E * slab * (bf16 ? 2 : 4);
+    if (bf16) {
+        static bool attr = false;
+        if (!attr) {
+            cudaError_t e = cudaFuncSetAttribute(unpermute_reduce_kernel<__nv_bfloat16>,
+                                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 (int)(UR_TOK * 64 * 4 + 64 * 512 * 2));
+            if (e != cudaSuccess) return e;
+            attr = true;
+        }
+        unpermute_reduce_kernel<__nv_bfloat16><<<grid, 256, smem, s>>>(
             (const __nv_bfloat16*)dx_perm, slot_of, dlogits, (const __nv_bfloat16*)w_router, po, P,
             (const __nv_bfloat16*)dx_sh, S, T, d, E, k, (__nv_bfloat16*)dx);
-    else
-        unpermute_reduce_kernel<float><<<blocks, 256, 0, s>>>(
+    } else {
+        static bool attr = false;
+        if (!attr) {
+            cudaError_t e = cudaFuncSetAttribute(unpermute_reduce_kernel<float>,
+                                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 (int)(UR_TOK * 64 * 4 + 64 * 256 * 4));
+            if (e != cudaSuccess) return e;
+            attr = true;
+        }
+        unpermute_reduce_kernel<float><<<grid, 256, smem, s>>>(
             (const float*)dx_perm, slot_of, dlogits, (const float*)w_router, po, P,
             (const float*)dx_sh, S, T, d, E, k, (float*)dx);
+    }
     return cudaGetLastError();
 }
 

@@ -24,7 +24,11 @@ namespace tc {
 constexpr int BM = 128;
 constexpr int BK = 64;  // 64 bf16 = 128 bytes = one 128B-swizzle row
 constexpr int STAGES = 4;
-constexpr int THREADS = 192;
+constexpr int EPI_WARPS = 4;
+constexpr int THREADS = 64 + 32 * EPI_WARPS;  // TMA warp, MMA warp, epilogue warps
+constexpr int EPI_BOX = 32;                     // TMA-store box: 32 columns x 32 rows (bf16)
+constexpr int EPI_BUF_BYTES = EPI_BOX * EPI_BOX * 2;
+constexpr int EPI_STAGE_BYTES = 3 * EPI_BUF_BYTES;  // per epilogue warp: up to 3 outputs
 constexpr int MAX_GROUPS = 128;
 
 struct Params {
@@ -41,6 +45,11 @@ struct Params {
     void* out1;
     const void* aux;
     uint64_t wait_ns;
+    // EPI_ROUTE: out0 = logits, out1 = probs (fp32 [T,E]), aux = bias [P,E] or null
+    int E, k, normalize, hist_n;
+    int32_t* topk_idx;
+    float* topk_w;
+    int32_t* counts;
 };
 
 // ------------------------------------------------------------------------ PTX helpers
@@ -99,6 +108,26 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
         "l"((uint64_t)map), "r"(bar), "r"(c0), "r"(c1)
         : "memory");
 }
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, uint32_t src, int c0, int c1) {
+    asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                     (uint64_t)map),
+                 "r"(src), "r"(c0), "r"(c1)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read0() {
+    asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+}
+__device__ __forceinline__ void bulk_wait0() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+__device__ __forceinline__ void fence_proxy_async() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+// 32 fp32 values -> 32 bf16 (64 bytes) at dst (16-byte aligned; shared or global)
+__device__ __forceinline__ void store_row32(__nv_bfloat16* dst, const float* v) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) Vec<__nv_bfloat16>::store(dst + 8 * i, v + 8 * i);
+}
+
 __device__ __forceinline__ void fence_before() {
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
 }
@@ -137,6 +166,38 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
     for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// 32 lanes x 16 consecutive fp32 columns of the accumulator
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float* v) {
+    uint32_t r[16];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+        "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+          "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+// 16-byte read-only load (the buffer is not written while the kernel runs)
+__device__ __forceinline__ uint4 ldg_nc(const __nv_bfloat16* ptr) {
+    uint4 r;
+    asm volatile("ld.global.nc.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+                 : "l"(ptr));
+    return r;
+}
+__device__ __forceinline__ void unpack8(uint4 u, float* v) {
+    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const float2 f = __bfloat1622float2(h[i]);
+        v[2 * i] = f.x;
+        v[2 * i + 1] = f.y;
+    }
+}
+
 // Shared-memory matrix descriptor, 128B swizzle, sm_100 family layout:
 // start>>4 [0,14), LBO>>4 [16,30), SBO>>4 [32,46), version 1 [46,48), swizzle 2 [61,64).
 __device__ __forceinline__ uint64_t smem_desc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
@@ -167,17 +228,95 @@ struct Tile {
     int last_rows;      // K-var: valid contraction rows in the last k-block (1..64)
 };
 
+// ------------------------------------------------------------------------ router epilogue
+// Gating of Alg. 7 for the token of this TMEM lane: the thread holds all BN >= E
+// logits of its token, adds the party's bias, writes logits and Softmax
+// probabilities, picks the k largest logits (equal logits: lower expert id first),
+// writes the gate weights p[I] (renormalised on request) and counts the picks.
+template <int BN>
+__device__ __forceinline__ void route_epilogue(const Params& p, const Tile& ti, int m, bool valid,
+                                               uint32_t tbase, int* hist) {
+    float z[BN];
+    if constexpr (BN == 16) {
+        tmem_ld16(tbase, z);
+    } else {
+#pragma unroll
+        for (int c = 0; c < BN / 32; ++c) tmem_ld32(tbase + 32 * c, z + 32 * c);
+    }
+    if (!valid) return;
+    const int E = p.E, k = p.k;
+    const int64_t t = ti.out_row + m;
+    const float* bias = (const float*)p.aux;
+    float mx = -3.402823466e38f;
+#pragma unroll
+    for (int e = 0; e < BN; ++e) {
+        if (e < E) {
+            if (bias) z[e] += bias[ti.g * E + e];
+            mx = fmaxf(mx, z[e]);
+        }
+    }
+    float sum = 0.f;
+#pragma unroll
+    for (int e = 0; e < BN; ++e)
+        if (e < E) sum += expf(z[e] - mx);
+    float* lg = (float*)p.out0 + t * E;
+    float* pr = (float*)p.out1 + t * E;
+#pragma unroll
+    for (int e = 0; e < BN; e += 4) {
+        if (e < E) {
+            *reinterpret_cast<float4*>(lg + e) = make_float4(z[e], z[e + 1], z[e + 2], z[e + 3]);
+            *reinterpret_cast<float4*>(pr + e) =
+                make_float4(expf(z[e] - mx) / sum, expf(z[e + 1] - mx) / sum,
+                            expf(z[e + 2] - mx) / sum, expf(z[e + 3] - mx) / sum);
+        }
+    }
+    uint64_t taken = 0;
+    float wsum = 0.f;
+    int sel[8];
+    float wsel[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+        sel[j] = 0;
+        wsel[j] = 0.f;
+        if (j < k) {
+            int bi = -1;
+            float bv = 0.f;
+#pragma unroll
+            for (int e = 0; e < BN; ++e) {
+                if (e < E && !((taken >> e) & 1ull) && (bi < 0 || z[e] > bv)) {
+                    bi = e;
+                    bv = z[e];
+                }
+            }
+            taken |= 1ull << bi;
+            sel[j] = bi;
+            wsel[j] = expf(bv - mx) / sum;
+            wsum += wsel[j];
+        }
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+        if (j < k) {
+            p.topk_idx[t * k + j] = sel[j];
+            p.topk_w[t * k + j] = p.normalize ? wsel[j] / wsum : wsel[j];
+            atomicAdd(&hist[ti.g * E + sel[j]], 1);
+        }
+    }
+}
+
 // ------------------------------------------------------------------------ the kernel
 template <int BN, bool B_MN, bool VAR_K, int EPI>
 __global__ void __launch_bounds__(THREADS, 1)
     grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA,
-                        const __grid_constant__ CUtensorMap tmB, const Params p) {
+                        const __grid_constant__ CUtensorMap tmB,
+                        const __grid_constant__ CUtensorMap tmO0,
+                        const __grid_constant__ CUtensorMap tmO1, const Params p) {
     constexpr bool A_MN = VAR_K;
     constexpr uint32_t A_BYTES = BM * BK * 2;
     constexpr uint32_t B_BYTES = BN * BK * 2;
     constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
     constexpr uint32_t IDESC = instr_desc<BN, A_MN, B_MN>();
-    constexpr int TMEM_COLS = 2 * BN;
+    constexpr int TMEM_COLS = (2 * BN <= 32) ? 32 : (2 * BN <= 64) ? 64 : (2 * BN <= 128) ? 128 : (2 * BN <= 256) ? 256 : 512;
 
     extern __shared__ uint8_t smem_raw[];
     __shared__ uint64_t bars[2 * STAGES + 5];
@@ -189,7 +328,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     volatile int* abort_flag = &s_abort;
 
     // group -> tile prefix
-    const int tiles_n = (EPI == EPI_SWIGLU_FWD) ? p.N / 256 : p.N / BN;
+    const int tiles_n = (EPI == EPI_SWIGLU_FWD) ? p.N / 256 : (EPI == EPI_ROUTE) ? 1 : p.N / BN;
     if (threadIdx.x == 0) {
         int acc = 0;
         for (int g = 0; g < p.G; ++g) {
@@ -252,6 +391,11 @@ __global__ void __launch_bounds__(THREADS, 1)
     const uint32_t raw_u32 = smem_u32(smem_raw);
     const uint32_t ring = raw_u32 + ((1024u - (raw_u32 & 1023u)) & 1023u);
     uint8_t* ring_ptr = smem_raw + (ring - raw_u32);
+    uint8_t* stage_out = ring_ptr + (size_t)STAGES * STAGE_BYTES;  // EPI_WARPS x EPI_STAGE_BYTES
+    int* route_hist = reinterpret_cast<int*>(stage_out);             // EPI_ROUTE has no staging
+    if constexpr (EPI == EPI_ROUTE) {
+        for (int i = threadIdx.x; i < p.hist_n; i += blockDim.x) route_hist[i] = 0;
+    }
     const uint32_t bar0 = smem_u32(&bars[0]);
     auto full_bar = [&](int s) { return bar0 + 8u * s; };
     auto empty_bar = [&](int s) { return bar0 + 8u * (STAGES + s); };
@@ -266,7 +410,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
         for (int a = 0; a < 2; ++a) {
             mbar_init(tfull_bar(a), 1);
-            mbar_init(tempty_bar(a), 128);
+            mbar_init(tempty_bar(a), 32 * EPI_WARPS);
         }
         mbar_init(drain_bar, 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -364,23 +508,31 @@ __global__ void __launch_bounds__(THREADS, 1)
                 }
                 const uint32_t sa = ring + stage * STAGE_BYTES;
                 const uint32_t sb = sa + A_BYTES;
+                // K-variable groups: the last k-block may hold contraction rows of the next
+                // group. Only K=16 steps that contain valid rows are issued, and inside the
+                // last of them the A rows past the group's end are zeroed (A alone suffices:
+                // their products with any finite B row vanish).
+                int ksteps = BK / 16;
                 if (VAR_K && kb == ti.k_iters - 1 && ti.last_rows < BK) {
-                    // contraction rows past the group's end belong to the next group:
-                    // zero them in every 64-row box of A and B before the MMA reads them
-                    const int nbox = BM / 64 + BN / 64;
-                    const int zero_bytes = (BK - ti.last_rows) * 128;
-                    uint8_t* base = ring_ptr + (size_t)stage * STAGE_BYTES;
-                    for (int b = 0; b < nbox; ++b) {
-                        uint4* z = reinterpret_cast<uint4*>(base + b * 8192 + ti.last_rows * 128);
-                        for (int i = lane; i < zero_bytes / 16; i += 32) z[i] = make_uint4(0, 0, 0, 0);
+                    ksteps = (ti.last_rows + 15) / 16;
+                    const int zr0 = ti.last_rows, zr1 = ksteps * 16;
+                    if (zr1 > zr0) {
+                        uint8_t* base = ring_ptr + (size_t)stage * STAGE_BYTES;
+                        const int per_box = (zr1 - zr0) * 8;  // 16-byte words
+#pragma unroll
+                        for (int b = 0; b < BM / 64; ++b) {
+                            uint4* z = reinterpret_cast<uint4*>(base + b * 8192 + zr0 * 128);
+                            for (int i = lane; i < per_box; i += 32) z[i] = make_uint4(0, 0, 0, 0);
+                        }
+                        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
                     }
-                    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
                     __syncwarp();
                 }
                 fence_after();
                 if (lane == 0) {
 #pragma unroll
                     for (int kk = 0; kk < BK / 16; ++kk) {
+                        if (kk >= ksteps) break;
                         uint64_t ad, bd;
                         if (!A_MN) ad = smem_desc(sa + kk * 32, 16, 1024);
                         else ad = smem_desc(sa + kk * 2048, 8192, 1024);
@@ -417,90 +569,140 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
         __syncwarp();
     } else {
-        // ------------------------------------------------------------ epilogue (warps 2-5)
-        const int q = warp & 3;  // TMEM lane quarter this warp may access
+        // ------------------------------------------------------------ epilogue warps 2-5
+        // Warp w reads TMEM lane quarter w % 4 (32 rows). Finished 32x32 bf16 boxes are
+        // staged in shared memory and written by TMA stores; a box that reaches past the
+        // group's last row (the last M tile of an expert) is written row by row instead.
+        const int q = warp & 3;
         const int row_local = q * 32 + lane;
+        uint8_t* stg = stage_out + (size_t)(warp - 2) * EPI_STAGE_BYTES;
+        const uint32_t stg_u32 = smem_u32(stg);
         int acc = 0;
         uint32_t acc_phase = 0;
         for (int t = blockIdx.x; t < total_tiles; t += gridDim.x) {
             const Tile ti = tile_at(t);
-            if (!mbar_wait(tfull_bar(acc), acc_phase, abort_flag, limit)) break;
-            fence_after();
-            const uint32_t tbase = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
             const int m = ti.m0 + row_local;
             const bool valid = m < ti.mvalid;
-            if (EPI == EPI_SWIGLU_FWD) {
+            const int wrow0 = ti.m0 + q * 32;
+            const bool full_box = wrow0 + 32 <= ti.mvalid;
+            const int64_t grow0 = VAR_K ? (int64_t)ti.g * p.Mout + wrow0 : ti.out_row + wrow0;
+            const uint32_t tbase = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
+            // write NOUT rows of 32 values each: staged + TMA when the whole box is valid
+            auto emit = [&](int nout, const float* const* vals, const CUtensorMap* const* maps,
+                            const int* cols, __nv_bfloat16* const* direct) {
+                if (full_box) {
+                    if (lane == 0) bulk_wait_read0();  // staging free again
+                    __syncwarp();
+                    for (int o = 0; o < nout; ++o)
+                        store_row32(reinterpret_cast<__nv_bfloat16*>(stg + o * EPI_BUF_BYTES + lane * 64), vals[o]);
+                    fence_proxy_async();
+                    __syncwarp();
+                    if (lane == 0) {
+                        for (int o = 0; o < nout; ++o)
+                            tma_store_2d(maps[o], stg_u32 + o * EPI_BUF_BYTES, cols[o], (int)grow0);
+                        bulk_commit();
+                    }
+                } else if (valid) {
+                    for (int o = 0; o < nout; ++o) store_row32(direct[o], vals[o]);
+                }
+            };
+            if constexpr (EPI == EPI_SWIGLU_BWD) {
+                // dA in TMEM; G and U come from h_gu. The next chunk's loads are in flight
+                // while the current one is computed; the first are issued before the wait.
                 const int F = p.F;
-                __nv_bfloat16* hgu = (__nv_bfloat16*)p.out0 + (ti.out_row + m) * (int64_t)(2 * F);
-                __nv_bfloat16* act = (__nv_bfloat16*)p.out1 + (ti.out_row + m) * (int64_t)F;
+                const __nv_bfloat16* __restrict__ hgu =
+                    (const __nv_bfloat16*)p.aux + (ti.out_row + m) * (int64_t)(2 * F) + ti.n0;
+                __nv_bfloat16* dh = (__nv_bfloat16*)p.out0 + (ti.out_row + m) * (int64_t)(2 * F) + ti.n0;
+                uint4 gc[4], uc[4];
+#pragma unroll
+                for (int v = 0; v < 4; ++v) {
+                    gc[v] = valid ? ldg_nc(hgu + 8 * v) : make_uint4(0, 0, 0, 0);
+                    uc[v] = valid ? ldg_nc(hgu + F + 8 * v) : make_uint4(0, 0, 0, 0);
+                }
+                if (!mbar_wait(tfull_bar(acc), acc_phase, abort_flag, limit)) break;
+                fence_after();
 #pragma unroll 1
-                for (int c = 0; c < 128; c += 32) {
-                    float g[32], u[32];
-                    tmem_ld32(tbase + c, g);
-                    tmem_ld32(tbase + 128 + c, u);
-                    if (valid) {
-                        const int f = ti.n0 + c;
+                for (int c = 0; c < BN / 32; ++c) {
+                    uint4 gn[4], un[4];
+                    if (c + 1 < BN / 32) {
 #pragma unroll
                         for (int v = 0; v < 4; ++v) {
-                            float a8[8];
-#pragma unroll
-                            for (int i = 0; i < 8; ++i) {
-                                const float G = g[8 * v + i], U = u[8 * v + i];
-                                a8[i] = G / (1.0f + expf(-G)) * U;
-                            }
-                            Vec<__nv_bfloat16>::store(hgu + f + 8 * v, g + 8 * v);
-                            Vec<__nv_bfloat16>::store(hgu + F + f + 8 * v, u + 8 * v);
-                            Vec<__nv_bfloat16>::store(act + f + 8 * v, a8);
+                            gn[v] = valid ? ldg_nc(hgu + 32 * (c + 1) + 8 * v) : make_uint4(0, 0, 0, 0);
+                            un[v] = valid ? ldg_nc(hgu + F + 32 * (c + 1) + 8 * v) : make_uint4(0, 0, 0, 0);
                         }
                     }
-                }
-            } else if (EPI == EPI_SWIGLU_BWD) {
-                const int F = p.F;
-                const __nv_bfloat16* hgu =
-                    (const __nv_bfloat16*)p.aux + (ti.out_row + m) * (int64_t)(2 * F);
-                __nv_bfloat16* dh = (__nv_bfloat16*)p.out0 + (ti.out_row + m) * (int64_t)(2 * F);
-#pragma unroll 1
-                for (int c = 0; c < BN; c += 32) {
-                    float da[32];
-                    tmem_ld32(tbase + c, da);
-                    if (valid) {
-                        const int f = ti.n0 + c;
+                    float da[32], dG[32], dU[32];
+                    tmem_ld32(tbase + 32 * c, da);
+#pragma unroll
+                    for (int v = 0; v < 4; ++v) {
+                        float G[8], U[8];
+                        unpack8(gc[v], G);
+                        unpack8(uc[v], U);
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) {
+                            const float sg = 1.0f / (1.0f + expf(-G[i]));
+                            const float d = da[8 * v + i];
+                            dU[8 * v + i] = d * G[i] * sg;
+                            dG[8 * v + i] = d * U[i] * sg * (1.0f + G[i] * (1.0f - sg));
+                        }
+                    }
+                    const float* vals[2] = {dG, dU};
+                    const CUtensorMap* maps[2] = {&tmO0, &tmO0};
+                    const int cols[2] = {ti.n0 + 32 * c, F + ti.n0 + 32 * c};
+                    __nv_bfloat16* direct[2] = {dh + 32 * c, dh + F + 32 * c};
+                    emit(2, vals, maps, cols, direct);
+                    if (c + 1 < BN / 32) {
 #pragma unroll
                         for (int v = 0; v < 4; ++v) {
-                            float G[8], U[8], dG[8], dU[8];
-                            Vec<__nv_bfloat16>::load(hgu + f + 8 * v, G);
-                            Vec<__nv_bfloat16>::load(hgu + F + f + 8 * v, U);
-#pragma unroll
-                            for (int i = 0; i < 8; ++i) {
-                                const float s = 1.0f / (1.0f + expf(-G[i]));
-                                const float d = da[8 * v + i];
-                                dU[i] = d * G[i] * s;
-                                dG[i] = d * U[i] * s * (1.0f + G[i] * (1.0f - s));
-                            }
-                            Vec<__nv_bfloat16>::store(dh + f + 8 * v, dG);
-                            Vec<__nv_bfloat16>::store(dh + F + f + 8 * v, dU);
+                            gc[v] = gn[v];
+                            uc[v] = un[v];
                         }
                     }
                 }
             } else {
-                __nv_bfloat16* out;
-                if (VAR_K)
-                    out = (__nv_bfloat16*)p.out0 + (int64_t)ti.g * p.Mout * p.N + (int64_t)m * p.N;
-                else
-                    out = (__nv_bfloat16*)p.out0 + (ti.out_row + m) * (int64_t)p.N;
+                if (!mbar_wait(tfull_bar(acc), acc_phase, abort_flag, limit)) break;
+                fence_after();
+                if constexpr (EPI == EPI_SWIGLU_FWD) {
+                    // accumulator columns [0,128) = G, [128,256) = U of features n0 .. n0+127
+                    const int F = p.F;
+                    __nv_bfloat16* hgu = (__nv_bfloat16*)p.out0 + (ti.out_row + m) * (int64_t)(2 * F);
+                    __nv_bfloat16* actp = (__nv_bfloat16*)p.out1 + (ti.out_row + m) * (int64_t)F;
 #pragma unroll 1
-                for (int c = 0; c < BN; c += 32) {
-                    float y[32];
-                    if (ti.k_iters > 0) {
-                        tmem_ld32(tbase + c, y);
-                    } else {
+                    for (int c = 0; c < 128; c += 32) {
+                        float g[32], u[32], a[32];
+                        tmem_ld32(tbase + c, g);
+                        tmem_ld32(tbase + 128 + c, u);
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) y[i] = 0.f;
+                        for (int i = 0; i < 32; ++i) a[i] = g[i] / (1.0f + expf(-g[i])) * u[i];
+                        const int f = ti.n0 + c;
+                        const float* vals[3] = {g, u, a};
+                        const CUtensorMap* maps[3] = {&tmO0, &tmO0, &tmO1};
+                        const int cols[3] = {f, F + f, f};
+                        __nv_bfloat16* direct[3] = {hgu + f, hgu + F + f, actp + f};
+                        emit(3, vals, maps, cols, direct);
                     }
-                    if (valid) {
+                } else if constexpr (EPI == EPI_ROUTE) {
+                    route_epilogue<BN>(p, ti, m, valid, tbase, route_hist);
+                } else {
+                    __nv_bfloat16* out;
+                    if (VAR_K)
+                        out = (__nv_bfloat16*)p.out0 + (int64_t)ti.g * p.Mout * p.N + (int64_t)m * p.N;
+                    else
+                        out = (__nv_bfloat16*)p.out0 + (ti.out_row + m) * (int64_t)p.N;
+#pragma unroll 1
+                    for (int c = 0; c < BN; c += 32) {
+                        float y[32];
+                        if (ti.k_iters > 0) {
+                            tmem_ld32(tbase + c, y);
+                        } else {
 #pragma unroll
-                        for (int v = 0; v < 4; ++v)
-                            Vec<__nv_bfloat16>::store(out + ti.n0 + c + 8 * v, y + 8 * v);
+                            for (int i = 0; i < 32; ++i) y[i] = 0.f;
+                        }
+                        const float* vals[1] = {y};
+                        const CUtensorMap* maps[1] = {&tmO0};
+                        const int cols[1] = {ti.n0 + c};
+                        __nv_bfloat16* direct[1] = {out + ti.n0 + c};
+                        emit(1, vals, maps, cols, direct);
                     }
                 }
             }
@@ -511,6 +713,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                 acc_phase ^= 1u;
             }
         }
+        if (lane == 0) bulk_wait0();  // every TMA store of this warp has completed
     }
     fence_before();
     __syncthreads();
@@ -519,6 +722,10 @@ __global__ void __launch_bounds__(THREADS, 1)
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base),
                      "r"(TMEM_COLS)
                      : "memory");
+    }
+    if constexpr (EPI == EPI_ROUTE) {
+        for (int i = threadIdx.x; i < p.hist_n; i += blockDim.x)
+            if (route_hist[i]) atomicAdd(&p.counts[i], route_hist[i]);
     }
 }
 
@@ -541,16 +748,19 @@ static EncodeTiledFn encode_fn() {
     return fn;
 }
 
-// 2D bf16 tensor [outer, inner] row-major, box {64, box_rows}, 128B swizzle, zero fill.
-static bool make_map(CUtensorMap* m, const void* base, int64_t inner, int64_t outer, int box_rows) {
+// 2D bf16 tensor [outer, inner] row-major, box {64, box_rows}, 128B swizzle, zero fill
+// (operand loads); with store = true a plain {32, 32} box for the epilogue's TMA stores.
+static bool make_map(CUtensorMap* m, const void* base, int64_t inner, int64_t outer, int box_rows,
+                     bool store = false) {
     EncodeTiledFn fn = encode_fn();
     if (!fn) return false;
     cuuint64_t dims[2] = {(cuuint64_t)inner, (cuuint64_t)outer};
     cuuint64_t strides[1] = {(cuuint64_t)inner * 2};
-    cuuint32_t box[2] = {64u, (cuuint32_t)box_rows};
+    cuuint32_t box[2] = {store ? (cuuint32_t)EPI_BOX : 64u, store ? (cuuint32_t)EPI_BOX : (cuuint32_t)box_rows};
     cuuint32_t estr[2] = {1u, 1u};
     CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
-                    box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                    box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                    store ? CU_TENSOR_MAP_SWIZZLE_NONE : CU_TENSOR_MAP_SWIZZLE_128B,
                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS;
 }
@@ -569,19 +779,23 @@ static int sm_count() {
 }
 
 template <int BN, bool B_MN, bool VAR_K, int EPI>
-static cudaError_t launch(const CUtensorMap& ma, const CUtensorMap& mb, const Params& p,
-                          int64_t tiles_ub, cudaStream_t s) {
+static cudaError_t launch(const CUtensorMap& ma, const CUtensorMap& mb, const CUtensorMap& mo0,
+                          const CUtensorMap& mo1, const Params& p, int64_t tiles_ub,
+                          cudaStream_t s) {
     auto kern = grouped_gemm_kernel<BN, B_MN, VAR_K, EPI>;
-    const int smem = STAGES * (BM * BK * 2 + BN * BK * 2) + 1024;
+    const int extra_max = EPI == EPI_ROUTE ? 64 * 64 * 4 : EPI_WARPS * EPI_STAGE_BYTES;
+    const int extra = EPI == EPI_ROUTE ? p.hist_n * 4 : EPI_WARPS * EPI_STAGE_BYTES;
+    const int smem_max = STAGES * (BM * BK * 2 + BN * BK * 2) + 1024 + extra_max;
+    const int smem = STAGES * (BM * BK * 2 + BN * BK * 2) + 1024 + extra;
     static bool attr_set = false;
     if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_max);
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
     if (tiles_ub <= 0) return cudaSuccess;
     const int grid = (int)std::min<int64_t>(tiles_ub, sm_count());
-    kern<<<grid, THREADS, smem, s>>>(ma, mb, p);
+    kern<<<grid, THREADS, smem, s>>>(ma, mb, mo0, mo1, p);
     return cudaGetLastError();
 }
 
@@ -612,34 +826,42 @@ cudaError_t launch_gemm_m(const GemmMArgs& g, bool bf16, cudaStream_t s) {
                                           : std::max<int64_t>(g.rows.rows, (int64_t)(g.G - 1) * g.rows.a_stride + g.rows.rows);
     const int64_t mt_ub = g.rows.offsets ? ((int64_t)g.rows.rows + BM - 1) / BM + g.G
                                          : (int64_t)g.G * ((g.rows.rows + BM - 1) / BM);
-    CUtensorMap ma, mb;
+    // output rows in the 2D view of the outputs
+    const int64_t o_rows = g.rows.offsets ? (int64_t)g.rows.rows
+                                          : std::max<int64_t>(g.rows.rows, (int64_t)(g.G - 1) * g.rows.out_stride + g.rows.rows);
+    CUtensorMap ma, mb, mo0, mo1;
     if (!make_map(&ma, g.a, g.K, a_rows, BM)) return cudaErrorInvalidValue;
     if (g.epi == EPI_SWIGLU_FWD) {
         const int F = g.N / 2;
         p.F = F;
         p.b_group_rows = 2 * (int64_t)F;
         if (!make_map(&mb, g.b, g.K, (int64_t)g.G * 2 * F, 128)) return cudaErrorInvalidValue;
-        return launch<256, false, false, EPI_SWIGLU_FWD>(ma, mb, p, mt_ub * (F / 128), s);
+        if (!make_map(&mo0, g.out0, 2 * (int64_t)F, o_rows, 0, true)) return cudaErrorInvalidValue;
+        if (!make_map(&mo1, g.out1, F, o_rows, 0, true)) return cudaErrorInvalidValue;
+        return launch<256, false, false, EPI_SWIGLU_FWD>(ma, mb, mo0, mo1, p, mt_ub * (F / 128), s);
     }
     if (g.epi == EPI_STORE && g.b_kmajor) {  // Y = A W2^T: B = W2[e] as [N=d, K=F]
         p.b_group_rows = g.N;
+        if (!make_map(&mo0, g.out0, g.N, o_rows, 0, true)) return cudaErrorInvalidValue;
         if (g.N % 256 == 0) {
             if (!make_map(&mb, g.b, g.K, (int64_t)g.G * g.N, 256)) return cudaErrorInvalidValue;
-            return launch<256, false, false, EPI_STORE>(ma, mb, p, mt_ub * (g.N / 256), s);
+            return launch<256, false, false, EPI_STORE>(ma, mb, mo0, mo0, p, mt_ub * (g.N / 256), s);
         }
         if (!make_map(&mb, g.b, g.K, (int64_t)g.G * g.N, 128)) return cudaErrorInvalidValue;
-        return launch<128, false, false, EPI_STORE>(ma, mb, p, mt_ub * (g.N / 128), s);
+        return launch<128, false, false, EPI_STORE>(ma, mb, mo0, mo0, p, mt_ub * (g.N / 128), s);
     }
     // MN-major B: weights stored [G*K, N]
     p.b_group_rows = g.K;
     if (!make_map(&mb, g.b, g.N, (int64_t)g.G * g.K, 64)) return cudaErrorInvalidValue;
     if (g.epi == EPI_SWIGLU_BWD) {
         p.F = g.N;
-        if (g.N % 256 == 0) return launch<256, true, false, EPI_SWIGLU_BWD>(ma, mb, p, mt_ub * (g.N / 256), s);
-        return launch<128, true, false, EPI_SWIGLU_BWD>(ma, mb, p, mt_ub * (g.N / 128), s);
+        if (!make_map(&mo0, g.out0, 2 * (int64_t)g.N, o_rows, 0, true)) return cudaErrorInvalidValue;
+        if (g.N % 256 == 0) return launch<256, true, false, EPI_SWIGLU_BWD>(ma, mb, mo0, mo0, p, mt_ub * (g.N / 256), s);
+        return launch<128, true, false, EPI_SWIGLU_BWD>(ma, mb, mo0, mo0, p, mt_ub * (g.N / 128), s);
     }
-    if (g.N % 256 == 0) return launch<256, true, false, EPI_STORE>(ma, mb, p, mt_ub * (g.N / 256), s);
-    return launch<128, true, false, EPI_STORE>(ma, mb, p, mt_ub * (g.N / 128), s);
+    if (!make_map(&mo0, g.out0, g.N, o_rows, 0, true)) return cudaErrorInvalidValue;
+    if (g.N % 256 == 0) return launch<256, true, false, EPI_STORE>(ma, mb, mo0, mo0, p, mt_ub * (g.N / 256), s);
+    return launch<128, true, false, EPI_STORE>(ma, mb, mo0, mo0, p, mt_ub * (g.N / 128), s);
 }
 
 // K-variable grouped GEMM (dW1, dW2).
@@ -661,12 +883,49 @@ cudaError_t launch_gemm_k(const GemmKArgs& g, bool bf16, cudaStream_t s) {
                                           : std::max<int64_t>(g.rows.rows, (int64_t)(g.G - 1) * g.rows.a_stride + g.rows.rows);
     const int64_t rows_b = g.rows.offsets ? (int64_t)g.rows.rows
                                           : std::max<int64_t>(g.rows.rows, (int64_t)(g.G - 1) * g.rows.b_stride + g.rows.rows);
-    CUtensorMap ma, mb;
+    CUtensorMap ma, mb, mo;
     if (!make_map(&ma, g.a, g.M, rows_a, 64)) return cudaErrorInvalidValue;
     if (!make_map(&mb, g.b, g.N, rows_b, 64)) return cudaErrorInvalidValue;
+    if (!make_map(&mo, g.out, g.N, (int64_t)g.G * g.M, 0, true)) return cudaErrorInvalidValue;
     const int64_t tiles = (int64_t)g.G * (g.M / BM);
-    if (g.N % 256 == 0) return launch<256, true, true, EPI_STORE>(ma, mb, p, tiles * (g.N / 256), s);
-    return launch<128, true, true, EPI_STORE>(ma, mb, p, tiles * (g.N / 128), s);
+    if (g.N % 256 == 0) return launch<256, true, true, EPI_STORE>(ma, mb, mo, mo, p, tiles * (g.N / 256), s);
+    return launch<128, true, true, EPI_STORE>(ma, mb, mo, mo, p, tiles * (g.N / 128), s);
+}
+
+// Router logits on the tensor cores with the gating epilogue: groups are parties
+// (rows [po[p], po[p+1]) use W_r[p]); N = E rounded up to 16, 32 or 64.
+cudaError_t launch_route_tc(const RouteArgs& a, cudaStream_t s) {
+    using namespace tc;
+    Params p{};
+    if (a.po && a.P > 1) {
+        p.offsets = a.po;
+        p.G = a.P;
+    } else {
+        p.rows = (int)a.T;
+        p.G = 1;
+    }
+    p.K = a.d;
+    p.E = a.E;
+    p.k = a.k;
+    p.normalize = a.normalize;
+    p.hist_n = a.P * a.E;
+    p.out0 = a.logits;
+    p.out1 = a.probs;
+    p.aux = a.bias;
+    p.topk_idx = a.topk_idx;
+    p.topk_w = a.topk_w;
+    p.counts = a.counts;
+    p.b_group_rows = a.E;
+    p.wait_ns = g_wait_ns;
+    const int BNr = a.E <= 16 ? 16 : a.E <= 32 ? 32 : 64;
+    p.N = BNr;
+    CUtensorMap ma, mb;
+    if (!make_map(&ma, a.x, a.d, a.T, BM)) return cudaErrorInvalidValue;
+    if (!make_map(&mb, a.w_router, a.d, (int64_t)a.P * a.E, BNr)) return cudaErrorInvalidValue;
+    const int64_t tiles = (a.T + BM - 1) / BM + a.P;
+    if (BNr == 16) return launch<16, false, false, EPI_ROUTE>(ma, mb, ma, ma, p, tiles, s);
+    if (BNr == 32) return launch<32, false, false, EPI_ROUTE>(ma, mb, ma, ma, p, tiles, s);
+    return launch<64, false, false, EPI_ROUTE>(ma, mb, ma, ma, p, tiles, s);
 }
 
 cudaError_t gemm_status(cudaStream_t s, int* code) { return tu_status_read_clear(s, code); }

@@ -40,6 +40,8 @@ struct RouteBwdArgs {
 };
 
 cudaError_t launch_route(const RouteArgs& a, bool bf16, bool from_logits, cudaStream_t s);
+// bf16 router logits on the tensor cores with the gating epilogue (E <= 64, E % 4 == 0)
+cudaError_t launch_route_tc(const RouteArgs& a, cudaStream_t s);
 cudaError_t launch_aux_loss(const float* probs, const int32_t* counts, const int32_t* po, int P,
                             int64_t T, int E, int k, float alpha, float* loss, float* coef,
                             cudaStream_t s);
@@ -71,7 +73,7 @@ cudaError_t launch_dispatch_noalloc(const int32_t* topk_idx, const void* x, int6
                                     int32_t* token_of, void* x_perm, cudaStream_t s);
 
 // grouped GEMMs -------------------------------------------------------------------------
-enum EpiKind { EPI_SWIGLU_FWD = 0, EPI_STORE = 1, EPI_SWIGLU_BWD = 2 };
+enum EpiKind { EPI_SWIGLU_FWD = 0, EPI_STORE = 1, EPI_SWIGLU_BWD = 2, EPI_ROUTE = 3 };
 
 // How the groups (experts) of a grouped GEMM are laid out along the rows that vary:
 //  OFFSETS: group g owns rows [offsets[g], offsets[g+1]) of A / out (M-variable) or of

@@ -3,10 +3,14 @@
 // vector loads, logits are reduced with warp shuffles, top-k is a warp argmax.
 #include <cfloat>
 
+#include <cooperative_groups.h>
+
 #include "moe_common.cuh"
 #include "moe_internal.h"
 
 namespace moe {
+
+namespace cg = cooperative_groups;
 
 // ----------------------------------------------------------------------------- top-k
 // Per token, lane l owns experts l and l + 32 (E <= 64). Picks the k largest logits,
@@ -166,38 +170,61 @@ __global__ void __launch_bounds__(256) route_kernel(
 }
 
 // ----------------------------------------------------------------------------- aux loss
-// One block per party; deterministic fixed-order reductions.
-__global__ void __launch_bounds__(256) aux_loss_kernel(const float* __restrict__ probs,
-                                                      const int32_t* __restrict__ counts,
-                                                      const int32_t* __restrict__ po, int64_t Tn,
-                                                      int E, int k, float alpha, float* loss,
-                                                      float* coef) {
-    __shared__ float s_part[256];
-    __shared__ float s_term[64];
-    const int p = blockIdx.x;
+// One 8-CTA thread-block cluster per party: each CTA sums probs[t, e] over its slice
+// of the party's tokens (fixed order inside the CTA), then CTA 0 of the cluster adds
+// the 8 partial rows from distributed shared memory in rank order. Deterministic,
+// no workspace, no floating-point atomics.
+constexpr int AUX_CLUSTER = 8;
+constexpr int AUX_THREADS = 1024;
+
+__global__ void __cluster_dims__(AUX_CLUSTER, 1, 1) __launch_bounds__(AUX_THREADS)
+    aux_loss_kernel(const float* __restrict__ probs, const int32_t* __restrict__ counts,
+                    const int32_t* __restrict__ po, int64_t Tn, int E, int k, float alpha,
+                    float* loss, float* coef) {
+    __shared__ float s_part[AUX_THREADS];
+    __shared__ float s_col[64];
+    cg::cluster_group cluster = cg::this_cluster();
+    const int rank = (int)cluster.block_rank();
+    const int p = blockIdx.x / AUX_CLUSTER;
     const int64_t a = po ? po[p] : 0, b = po ? po[p + 1] : Tn;
-    const int lpe = blockDim.x / E;  // stripes per expert
+    const int64_t n = b - a;
+    const int64_t per = (n + AUX_CLUSTER - 1) / AUX_CLUSTER;
+    const int64_t lo = a + min64(n, per * rank), hi = a + min64(n, per * (rank + 1));
     const int tid = threadIdx.x;
-    float s = 0.f;
-    if (tid < lpe * E) {
-        const int e = tid % E, stripe = tid / E;
-        for (int64_t t = a + stripe; t < b; t += lpe) s += probs[t * E + e];
+    const int stripes = AUX_THREADS / E;
+    float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+    if (tid < stripes * E) {
+        const int e = tid % E, st = tid / E;
+        int64_t t = lo + st;
+        for (; t + 3 * stripes < hi; t += 4 * stripes) {
+            s0 += probs[t * E + e];
+            s1 += probs[(t + stripes) * E + e];
+            s2 += probs[(t + 2 * stripes) * E + e];
+            s3 += probs[(t + 3 * stripes) * E + e];
+        }
+        for (; t < hi; t += stripes) s0 += probs[t * E + e];
     }
-    s_part[tid] = s;
+    s_part[tid] = (s0 + s1) + (s2 + s3);
     __syncthreads();
     if (tid < E) {
         float tot = 0.f;
-        for (int st = 0; st < lpe; ++st) tot += s_part[st * E + tid];
-        const float Tp = (float)(b - a);
-        const float f = (Tp > 0) ? (float)counts[p * E + tid] / (Tp * k) : 0.f;
-        const float Pm = (Tp > 0) ? tot / Tp : 0.f;
-        s_term[tid] = f * Pm;
-        coef[p * E + tid] = (Tp > 0) ? alpha * E * f / Tp : 0.f;
+        for (int st = 0; st < stripes; ++st) tot += s_part[st * E + tid];
+        s_col[tid] = tot;
     }
-    __syncthreads();
-    if (tid == 0) {
+    cluster.sync();
+    if (rank == 0 && tid < E) {
+        float tot = 0.f;
+        for (int r = 0; r < AUX_CLUSTER; ++r) tot += cluster.map_shared_rank(s_col, r)[tid];
+        const float Tp = (float)n;
+        const float f = (n > 0) ? (float)counts[p * E + tid] / (Tp * k) : 0.f;
+        const float Pm = (n > 0) ? tot / Tp : 0.f;
+        s_part[tid] = f * Pm;
+        coef[p * E + tid] = (n > 0) ? alpha * E * f / Tp : 0.f;
+    }
+    cluster.sync();
+    if (rank == 0 && tid == 0) {
         float L = 0.f;
-        for (int e = 0; e < E; ++e) L += s_term[e];
+        for (int e = 0; e < E; ++e) L += s_part[e];
         loss[p] = alpha * E * L;
     }
 }
@@ -220,16 +247,22 @@ __device__ __forceinline__ bool chunk_of(int64_t ci, const int32_t* po, int P, i
     return false;
 }
 
-// dlogits of one token (lane l: experts l, l+32), Alg. 7 backward with fixed picks.
-__device__ __forceinline__ void dlogits_token(int64_t t, int lane, int E, int k, int normalize,
-                                              int party, const float* probs,
-                                              const int32_t* topk_idx, const float* topk_w,
-                                              const float* dtopk_w, const float* aux_coef,
-                                              float* dz0, float* dz1) {
-    const int e0 = lane, e1 = lane + 32;
-    float p0 = e0 < E ? probs[t * E + e0] : 0.f;
-    float p1 = e1 < E ? probs[t * E + e1] : 0.f;
-    float dp0 = 0.f, dp1 = 0.f;
+// dlogits, one thread per token (Alg. 7 backward with the picks held fixed).
+template <int EMAX>
+__global__ void __launch_bounds__(256) dlogits_kernel(
+    const float* __restrict__ probs, const int32_t* __restrict__ topk_idx,
+    const float* __restrict__ topk_w, const float* __restrict__ dtopk_w,
+    const float* __restrict__ aux_coef, const int32_t* __restrict__ po, int P, int64_t Tn, int E,
+    int k, int normalize, float* dlogits) {
+    const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (t >= Tn) return;
+    const int party = party_of(po, P, t);
+    float pr[EMAX], dp[EMAX];
+#pragma unroll
+    for (int e = 0; e < EMAX; ++e) {
+        pr[e] = (e < E) ? probs[t * E + e] : 0.f;
+        dp[e] = (e < E && aux_coef) ? aux_coef[party * E + e] : 0.f;
+    }
     float inner = 0.f, S = 0.f;
     if (normalize) {
         for (int j = 0; j < k; ++j) {
@@ -242,95 +275,110 @@ __device__ __forceinline__ void dlogits_token(int64_t t, int lane, int E, int k,
         const int e = topk_idx[t * k + j];
         float g = dtopk_w[t * k + j];
         if (normalize) g = (g - inner) / S;
-        if (e == e0) dp0 += g;
-        if (e == e1) dp1 += g;
+#pragma unroll
+        for (int q = 0; q < EMAX; ++q)
+            if (q == e) dp[q] += g;
     }
-    if (aux_coef) {
-        if (e0 < E) dp0 += aux_coef[party * E + e0];
-        if (e1 < E) dp1 += aux_coef[party * E + e1];
-    }
-    const float dot = warp_sum(dp0 * p0 + dp1 * p1);
-    *dz0 = p0 * (dp0 - dot);
-    *dz1 = p1 * (dp1 - dot);
+    float dot = 0.f;
+#pragma unroll
+    for (int e = 0; e < EMAX; ++e) dot = fmaf(dp[e], pr[e], dot);
+#pragma unroll
+    for (int e = 0; e < EMAX; ++e)
+        if (e < E) dlogits[t * E + e] = pr[e] * (dp[e] - dot);
 }
 
-// Stage A: per (token chunk, 8-expert tile, 1024-column slab): dlogits of the chunk
-// into shared memory (and to global once), then partial dW_r = dz^T x and partial db.
-constexpr int RB_CH = 64;    // tokens per chunk
-constexpr int RB_ET = 8;     // experts per tile
-constexpr int RB_COLS = 1024;
+// Partial dW_r = dlogits^T x and db over one chunk of RB_CH tokens of one party, for
+// a tile of RB_ET experts and a column slab. The two thread halves take alternate
+// tokens of the chunk and are added in a fixed order at the end.
+constexpr int RB_CH = 32;   // tokens per chunk
+constexpr int RB_ET = 16;   // experts per tile
+constexpr int RB_HALF = 128;  // threads per half
 
 template <typename T>
-__global__ void __launch_bounds__(128) route_bwd_partial_kernel(
-    const T* __restrict__ x, const float* __restrict__ probs, const int32_t* __restrict__ topk_idx,
-    const float* __restrict__ topk_w, const float* __restrict__ dtopk_w,
-    const float* __restrict__ aux_coef, const int32_t* __restrict__ po, int P, int64_t Tn, int d,
-    int E, int k, int normalize, float* dlogits, float* part_dw, float* part_db) {
-    __shared__ float s_dz[RB_CH][64];
+__global__ void __launch_bounds__(2 * RB_HALF) route_bwd_partial_kernel(
+    const T* __restrict__ x, const float* __restrict__ dz, const int32_t* __restrict__ po, int P,
+    int64_t Tn, int d, int E, float* part_dw, float* part_db) {
+    constexpr int VN = Vec<T>::N;
+    constexpr int SLAB = RB_HALF * VN;
+    __shared__ float s_dz[RB_CH][RB_ET];
+    extern __shared__ float s_acc[];  // [RB_HALF][RB_ET][VN]: the second half's sums
     int party, n;
     int64_t t0;
     if (!chunk_of(blockIdx.x, po, P, Tn, RB_CH, &party, &t0, &n)) return;
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const bool writer = (blockIdx.y == 0 && blockIdx.z == 0);
-    for (int i = warp; i < RB_CH; i += blockDim.x >> 5) {
-        float dz0 = 0.f, dz1 = 0.f;
-        if (i < n) {
-            dlogits_token(t0 + i, lane, E, k, normalize, party, probs, topk_idx, topk_w, dtopk_w,
-                          aux_coef, &dz0, &dz1);
-            if (writer) {
-                if (lane < E) dlogits[(t0 + i) * E + lane] = dz0;
-                if (lane + 32 < E) dlogits[(t0 + i) * E + lane + 32] = dz1;
-            }
-        }
-        s_dz[i][lane] = dz0;
-        s_dz[i][lane + 32] = dz1;
+    const int e0 = blockIdx.y * RB_ET;
+    const int ne = min(RB_ET, E - e0);
+    for (int i = threadIdx.x; i < RB_CH * RB_ET; i += blockDim.x) {
+        const int tt = i / RB_ET, e = i % RB_ET;
+        s_dz[tt][e] = (tt < n && e < ne) ? dz[(t0 + tt) * E + e0 + e] : 0.f;
     }
     __syncthreads();
-    const int e0 = blockIdx.y * RB_ET;
-    if (blockIdx.z == 0 && threadIdx.x < RB_ET && e0 + threadIdx.x < E) {
-        float s = 0.f;
-        for (int i = 0; i < n; ++i) s += s_dz[i][e0 + threadIdx.x];
-        part_db[(int64_t)blockIdx.x * E + e0 + threadIdx.x] = s;
+    const int half = threadIdx.x / RB_HALF, ht = threadIdx.x % RB_HALF;
+    if (blockIdx.z == 0 && threadIdx.x < ne) {
+        float sdb = 0.f;
+        for (int i = 0; i < n; ++i) sdb += s_dz[i][threadIdx.x];
+        part_db[(int64_t)blockIdx.x * E + e0 + threadIdx.x] = sdb;
     }
-    using V = Vec<T>;
-    constexpr int VN = V::N;
-    const int64_t c0 = (int64_t)blockIdx.z * RB_COLS + threadIdx.x * VN;
-    for (int64_t c = c0; c < min64(d, (int64_t)(blockIdx.z + 1) * RB_COLS); c += blockDim.x * VN) {
-        float acc[RB_ET][VN];
+    const int64_t c = (int64_t)blockIdx.z * SLAB + ht * VN;
+    const bool active = c < d;
+    float acc[RB_ET][VN];
+#pragma unroll
+    for (int e = 0; e < RB_ET; ++e)
+#pragma unroll
+        for (int q = 0; q < VN; ++q) acc[e][q] = 0.f;
+    if (active) {
+        // four tokens' x vectors are loaded before any of them is used
+        for (int i0 = half; i0 < n; i0 += 8) {
+            uint4 raw[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int i = i0 + 2 * u;
+                if (i < n) raw[u] = Vec<T>::raw_load(x + (t0 + i) * d + c);
+            }
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int i = i0 + 2 * u;
+                if (i >= n) break;
+                float xv[VN];
+                unpack_vec<T>(raw[u], xv);
+#pragma unroll
+                for (int e = 0; e < RB_ET; ++e) {
+                    const float zz = s_dz[i][e];
+#pragma unroll
+                    for (int q = 0; q < VN; ++q) acc[e][q] = fmaf(zz, xv[q], acc[e][q]);
+                }
+            }
+        }
+    }
+    if (half == 1) {
 #pragma unroll
         for (int e = 0; e < RB_ET; ++e)
 #pragma unroll
-            for (int q = 0; q < VN; ++q) acc[e][q] = 0.f;
-        for (int i = 0; i < n; ++i) {
-            float xv[VN];
-            V::load(x + (t0 + i) * d + c, xv);
-#pragma unroll
-            for (int e = 0; e < RB_ET; ++e) {
-                const float z = s_dz[i][(e0 + e) & 63];
-#pragma unroll
-                for (int q = 0; q < VN; ++q) acc[e][q] = fmaf(z, xv[q], acc[e][q]);
-            }
-        }
+            for (int q = 0; q < VN; ++q) s_acc[(ht * RB_ET + e) * VN + q] = acc[e][q];
+    }
+    __syncthreads();
+    if (half == 0 && active) {
 #pragma unroll
         for (int e = 0; e < RB_ET; ++e) {
-            if (e0 + e < E) {
+            if (e < ne) {
                 float* dst = part_dw + ((int64_t)blockIdx.x * E + e0 + e) * d + c;
+                float r[VN];
 #pragma unroll
-                for (int q = 0; q < VN; ++q) dst[q] = acc[e][q];
+                for (int q = 0; q < VN; ++q) r[q] = acc[e][q] + s_acc[(ht * RB_ET + e) * VN + q];
+                Vec<float>::store(dst, r);
+                if (VN == 8) Vec<float>::store(dst + 4, r + 4);
             }
         }
     }
 }
 
-// Stage B: sum the partials of each party's chunks in chunk order.
+// Sum the partials of each party's chunks in chunk order (four interleaved running
+// sums, combined in a fixed order).
 template <typename T>
 __global__ void __launch_bounds__(256) route_bwd_reduce_kernel(
     const float* __restrict__ part_dw, const float* __restrict__ part_db,
     const int32_t* __restrict__ po, int P, int64_t Tn, int d, int E, T* dw_router, float* dbias) {
     const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     const int64_t per_party = (int64_t)E * d;
-    const int64_t total = (int64_t)P * per_party;
-    // chunk range of party p
     auto crange = [&](int p, int64_t* first, int64_t* cnt) {
         int64_t base = 0;
         for (int q = 0; q < P; ++q) {
@@ -340,22 +388,30 @@ __global__ void __launch_bounds__(256) route_bwd_reduce_kernel(
             base += nc;
         }
     };
-    if (i < total) {
+    if (i < (int64_t)P * per_party) {
         const int p = (int)(i / per_party);
-        const int64_t rem = i % per_party;  // e*d + c
+        const int64_t rem = i % per_party;
         int64_t first, cnt;
         crange(p, &first, &cnt);
-        float s = 0.f;
-        for (int64_t c = 0; c < cnt; ++c) s += part_dw[(first + c) * per_party + rem];
-        Elem<T>::store(dw_router + i, s);
+        const float* src = part_dw + first * per_party + rem;
+        float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+        int64_t c = 0;
+        for (; c + 3 < cnt; c += 4) {
+            s0 += src[c * per_party];
+            s1 += src[(c + 1) * per_party];
+            s2 += src[(c + 2) * per_party];
+            s3 += src[(c + 3) * per_party];
+        }
+        for (; c < cnt; ++c) s0 += src[c * per_party];
+        Elem<T>::store(dw_router + i, (s0 + s1) + (s2 + s3));
     }
     if (dbias && i < (int64_t)P * E) {
         const int p = (int)(i / E), e = (int)(i % E);
         int64_t first, cnt;
         crange(p, &first, &cnt);
-        float s = 0.f;
-        for (int64_t c = 0; c < cnt; ++c) s += part_db[(first + c) * E + e];
-        dbias[i] = s;
+        float sum = 0.f;
+        for (int64_t c = 0; c < cnt; ++c) sum += part_db[(first + c) * E + e];
+        dbias[i] = sum;
     }
 }
 
@@ -403,13 +459,14 @@ cudaError_t launch_route(const RouteArgs& a, bool bf16, bool from_logits, cudaSt
     cudaError_t e = cudaMemsetAsync(a.counts, 0, sizeof(int32_t) * a.P * a.E, s);
     if (e != cudaSuccess) return e;
     if (from_logits) return launch_route_t<float, true>(a, s);
+    if (bf16 && a.E % 4 == 0 && a.T > 0) return launch_route_tc(a, s);
     return bf16 ? launch_route_t<__nv_bfloat16, false>(a, s) : launch_route_t<float, false>(a, s);
 }
 
 cudaError_t launch_aux_loss(const float* probs, const int32_t* counts, const int32_t* po, int P,
                             int64_t T, int E, int k, float alpha, float* loss, float* coef,
                             cudaStream_t s) {
-    aux_loss_kernel<<<P, 256, 0, s>>>(probs, counts, po, T, E, k, alpha, loss, coef);
+    aux_loss_kernel<<<P * AUX_CLUSTER, AUX_THREADS, 0, s>>>(probs, counts, po, T, E, k, alpha, loss, coef);
     return cudaGetLastError();
 }
 
@@ -423,10 +480,32 @@ static cudaError_t launch_route_bwd_t(const RouteBwdArgs& a, void* ws, cudaStrea
     const int64_t nch = (a.T + RB_CH - 1) / RB_CH + a.P;
     float* part_dw = (float*)ws;
     float* part_db = part_dw + nch * a.E * a.d;
-    dim3 grid((unsigned)nch, (a.E + RB_ET - 1) / RB_ET, (a.d + RB_COLS - 1) / RB_COLS);
-    route_bwd_partial_kernel<T><<<grid, 128, 0, s>>>(
-        (const T*)a.x, a.probs, a.topk_idx, a.topk_w, a.dtopk_w, a.aux_coef, a.po, a.P, a.T, a.d,
-        a.E, a.k, a.normalize, a.dlogits, part_dw, part_db);
+    if (a.T > 0) {
+        const unsigned blocks = (unsigned)((a.T + 63) / 64);
+#define MOE_DZ(EM)                                                                             \
+    dlogits_kernel<EM><<<blocks, 64, 0, s>>>(a.probs, a.topk_idx, a.topk_w, a.dtopk_w,        \
+                                              a.aux_coef, a.po, a.P, a.T, a.E, a.k,            \
+                                              a.normalize, a.dlogits)
+        if (a.E <= 8) MOE_DZ(8);
+        else if (a.E <= 16) MOE_DZ(16);
+        else if (a.E <= 32) MOE_DZ(32);
+        else MOE_DZ(64);
+#undef MOE_DZ
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
+    constexpr int SLAB = RB_HALF * Vec<T>::N;
+    dim3 grid((unsigned)nch, (a.E + RB_ET - 1) / RB_ET, (a.d + SLAB - 1) / SLAB);
+    const size_t smem = (size_t)RB_HALF * RB_ET * Vec<T>::N * sizeof(float);
+    static bool attr = false;
+    if (!attr) {
+        cudaError_t e = cudaFuncSetAttribute(route_bwd_partial_kernel<T>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        attr = true;
+    }
+    route_bwd_partial_kernel<T><<<grid, 2 * RB_HALF, smem, s>>>((const T*)a.x, a.dlogits, a.po,
+                                                                a.P, a.T, a.d, a.E, part_dw, part_db);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     const int64_t total = (int64_t)a.P * a.E * a.d;
