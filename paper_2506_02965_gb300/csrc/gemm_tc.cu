@@ -128,6 +128,15 @@ __device__ __forceinline__ void store_row32(__nv_bfloat16* dst, const float* v) 
     for (int i = 0; i < 4; ++i) Vec<__nv_bfloat16>::store(dst + 8 * i, v + 8 * i);
 }
 
+// One 64-byte row (32 bf16) of a staging box in the 64B-swizzled layout the TMA store
+// map uses: 16-byte chunk c of row r sits at chunk c ^ ((r >> 1) & 3).
+__device__ __forceinline__ void store_row32_sw64(uint8_t* row_base, int r, const float* v) {
+#pragma unroll
+    for (int c = 0; c < 4; ++c)
+        Vec<__nv_bfloat16>::store(reinterpret_cast<__nv_bfloat16*>(row_base + ((c ^ ((r >> 1) & 3)) << 4)),
+                                  v + 8 * c);
+}
+
 __device__ __forceinline__ void fence_before() {
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
 }
@@ -594,7 +603,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                     if (lane == 0) bulk_wait_read0();  // staging free again
                     __syncwarp();
                     for (int o = 0; o < nout; ++o)
-                        store_row32(reinterpret_cast<__nv_bfloat16*>(stg + o * EPI_BUF_BYTES + lane * 64), vals[o]);
+                        store_row32_sw64(stg + o * EPI_BUF_BYTES + lane * 64, lane, vals[o]);
                     fence_proxy_async();
                     __syncwarp();
                     if (lane == 0) {
@@ -640,7 +649,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                         unpack8(uc[v], U);
 #pragma unroll
                         for (int i = 0; i < 8; ++i) {
-                            const float sg = 1.0f / (1.0f + expf(-G[i]));
+                            const float sg = __fdividef(1.0f, 1.0f + __expf(-G[i]));
                             const float d = da[8 * v + i];
                             dU[8 * v + i] = d * G[i] * sg;
                             dG[8 * v + i] = d * U[i] * sg * (1.0f + G[i] * (1.0f - sg));
@@ -673,7 +682,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                         tmem_ld32(tbase + c, g);
                         tmem_ld32(tbase + 128 + c, u);
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) a[i] = g[i] / (1.0f + expf(-g[i])) * u[i];
+                        for (int i = 0; i < 32; ++i) a[i] = __fdividef(g[i], 1.0f + __expf(-g[i])) * u[i];
                         const int f = ti.n0 + c;
                         const float* vals[3] = {g, u, a};
                         const CUtensorMap* maps[3] = {&tmO0, &tmO0, &tmO1};
@@ -749,7 +758,7 @@ static EncodeTiledFn encode_fn() {
 }
 
 // 2D bf16 tensor [outer, inner] row-major, box {64, box_rows}, 128B swizzle, zero fill
-// (operand loads); with store = true a plain {32, 32} box for the epilogue's TMA stores.
+// (operand loads); with store = true a {32, 32} box, 64B swizzle, for the epilogue's TMA stores.
 static bool make_map(CUtensorMap* m, const void* base, int64_t inner, int64_t outer, int box_rows,
                      bool store = false) {
     EncodeTiledFn fn = encode_fn();
@@ -760,7 +769,7 @@ static bool make_map(CUtensorMap* m, const void* base, int64_t inner, int64_t ou
     cuuint32_t estr[2] = {1u, 1u};
     CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
                     box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                    store ? CU_TENSOR_MAP_SWIZZLE_NONE : CU_TENSOR_MAP_SWIZZLE_128B,
+                    store ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B,
                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS;
 }
