@@ -117,10 +117,8 @@ __global__ void __launch_bounds__(256) gather_kernel(const T* __restrict__ x,
 // out[t] = sum_j w[t,j] * y_perm[slot_of[t,j]] (+ sum_s y_sh[s,t]); fp32 accumulation.
 // One warp per token; every lane issues the loads of up to UB vectors of all k rows
 // before it uses any of them, so enough bytes are in flight to keep HBM busy.
-constexpr int UB = 4;
-
-template <typename T>
-__global__ void __launch_bounds__(256) combine_fwd_kernel(const T* __restrict__ y_perm,
+template <typename T, int KMAX>
+__global__ void __launch_bounds__(256, 3) combine_fwd_kernel(const T* __restrict__ y_perm,
                                                           const float* __restrict__ w,
                                                           const int32_t* __restrict__ slot_of,
                                                           const T* __restrict__ y_sh, int S,
@@ -129,10 +127,11 @@ __global__ void __launch_bounds__(256) combine_fwd_kernel(const T* __restrict__ 
     const int64_t t = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
     if (t >= Tn) return;
     constexpr int VN = Vec<T>::N;
-    int64_t slot[8];
-    float wt[8];
+    constexpr int UB = KMAX <= 2 ? 4 : KMAX <= 4 ? 2 : 1;  // vectors per lane in flight
+    int64_t slot[KMAX];
+    float wt[KMAX];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
+    for (int j = 0; j < KMAX; ++j) {
         slot[j] = j < k ? slot_of[t * k + j] : 0;
         wt[j] = j < k ? w[t * k + j] : 0.f;
         if (slot[j] < 0 || slot[j] >= Tn * k) {  // bad table: contribute nothing
@@ -143,12 +142,12 @@ __global__ void __launch_bounds__(256) combine_fwd_kernel(const T* __restrict__ 
     }
     const int nv = d / VN;
     for (int v0 = lane; v0 < nv; v0 += 32 * UB) {
-        uint4 raw[UB][8];
+        uint4 raw[UB][KMAX];
 #pragma unroll
         for (int u = 0; u < UB; ++u) {
             const int v = v0 + 32 * u;
 #pragma unroll
-            for (int j = 0; j < 8; ++j)
+            for (int j = 0; j < KMAX; ++j)
                 if (j < k && v < nv) raw[u][j] = Vec<T>::raw_load(y_perm + slot[j] * d + v * VN);
         }
 #pragma unroll
@@ -159,7 +158,7 @@ __global__ void __launch_bounds__(256) combine_fwd_kernel(const T* __restrict__ 
 #pragma unroll
             for (int q = 0; q < VN; ++q) acc[q] = 0.f;
 #pragma unroll
-            for (int j = 0; j < 8; ++j) {
+            for (int j = 0; j < KMAX; ++j) {
                 if (j < k) {
                     float yv[VN];
                     unpack_vec<T>(raw[u][j], yv);
@@ -179,8 +178,8 @@ __global__ void __launch_bounds__(256) combine_fwd_kernel(const T* __restrict__ 
 }
 
 // dy_perm[slot(t,j)] = w[t,j] dout[t];  dw[t,j] = <dout[t], y_perm[slot(t,j)]>.
-template <typename T>
-__global__ void __launch_bounds__(256) combine_bwd_kernel(const T* __restrict__ dout,
+template <typename T, int KMAX>
+__global__ void __launch_bounds__(256, 3) combine_bwd_kernel(const T* __restrict__ dout,
                                                           const T* __restrict__ y_perm,
                                                           const float* __restrict__ w,
                                                           const int32_t* __restrict__ slot_of,
@@ -190,10 +189,11 @@ __global__ void __launch_bounds__(256) combine_bwd_kernel(const T* __restrict__ 
     const int64_t t = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
     if (t >= Tn) return;
     constexpr int VN = Vec<T>::N;
-    int64_t slot[8];
-    float wt[8], part[8];
+    constexpr int UB = KMAX <= 2 ? 4 : KMAX <= 4 ? 2 : 1;
+    int64_t slot[KMAX];
+    float wt[KMAX], part[KMAX];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
+    for (int j = 0; j < KMAX; ++j) {
         slot[j] = j < k ? slot_of[t * k + j] : 0;
         wt[j] = j < k ? w[t * k + j] : 0.f;
         part[j] = 0.f;
@@ -204,14 +204,14 @@ __global__ void __launch_bounds__(256) combine_bwd_kernel(const T* __restrict__ 
     }
     const int nv = d / VN;
     for (int v0 = lane; v0 < nv; v0 += 32 * UB) {
-        uint4 graw[UB], yraw[UB][8];
+        uint4 graw[UB], yraw[UB][KMAX];
 #pragma unroll
         for (int u = 0; u < UB; ++u) {
             const int v = v0 + 32 * u;
             if (v < nv) {
                 graw[u] = Vec<T>::raw_load(dout + t * d + v * VN);
 #pragma unroll
-                for (int j = 0; j < 8; ++j)
+                for (int j = 0; j < KMAX; ++j)
                     if (j < k && slot[j] >= 0) yraw[u][j] = Vec<T>::raw_load(y_perm + slot[j] * d + v * VN);
             }
         }
@@ -222,7 +222,7 @@ __global__ void __launch_bounds__(256) combine_bwd_kernel(const T* __restrict__ 
             float g[VN];
             unpack_vec<T>(graw[u], g);
 #pragma unroll
-            for (int j = 0; j < 8; ++j) {
+            for (int j = 0; j < KMAX; ++j) {
                 if (j < k && slot[j] >= 0) {
                     float yv[VN], dy[VN];
                     unpack_vec<T>(yraw[u][j], yv);
@@ -237,7 +237,7 @@ __global__ void __launch_bounds__(256) combine_bwd_kernel(const T* __restrict__ 
         }
     }
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
+    for (int j = 0; j < KMAX; ++j) {
         if (j < k) {
             const float sum = warp_sum(part[j]);
             if (lane == 0) dw[t * k + j] = sum;
@@ -249,7 +249,7 @@ __global__ void __launch_bounds__(256) combine_bwd_kernel(const T* __restrict__ 
 // A block takes UR_TOK tokens of one party and a slab of 64 * VN columns: the party's
 // router rows for the slab and the tokens' dlogits are staged in shared memory; each
 // thread owns VN columns of UR_TOK / 4 tokens.
-constexpr int UR_TOK = 32;
+constexpr int UR_TOK = 16;
 
 template <typename T>
 __global__ void __launch_bounds__(256) unpermute_reduce_kernel(
@@ -382,13 +382,19 @@ cudaError_t launch_combine_fwd(const void* y_perm, const float* topk_w, const in
                                void* out, cudaStream_t s) {
     if (T == 0) return cudaSuccess;
     const unsigned blocks = (unsigned)((T + 7) / 8);
-    if (bf16)
-        combine_fwd_kernel<__nv_bfloat16><<<blocks, 256, 0, s>>>(
-            (const __nv_bfloat16*)y_perm, topk_w, slot_of, (const __nv_bfloat16*)y_sh, S, T, d, k,
-            (__nv_bfloat16*)out);
-    else
-        combine_fwd_kernel<float><<<blocks, 256, 0, s>>>((const float*)y_perm, topk_w, slot_of,
-                                                         (const float*)y_sh, S, T, d, k, (float*)out);
+#define MOE_CF(TT, KM)                                                                           \
+    combine_fwd_kernel<TT, KM><<<blocks, 256, 0, s>>>((const TT*)y_perm, topk_w, slot_of,         \
+                                                      (const TT*)y_sh, S, T, d, k, (TT*)out)
+    if (bf16) {
+        if (k <= 2) MOE_CF(__nv_bfloat16, 2);
+        else if (k <= 4) MOE_CF(__nv_bfloat16, 4);
+        else MOE_CF(__nv_bfloat16, 8);
+    } else {
+        if (k <= 2) MOE_CF(float, 2);
+        else if (k <= 4) MOE_CF(float, 4);
+        else MOE_CF(float, 8);
+    }
+#undef MOE_CF
     return cudaGetLastError();
 }
 
@@ -397,14 +403,19 @@ cudaError_t launch_combine_bwd(const void* dout, const void* y_perm, const float
                                void* dy_perm, float* dtopk_w, cudaStream_t s) {
     if (T == 0) return cudaSuccess;
     const unsigned blocks = (unsigned)((T + 7) / 8);
-    if (bf16)
-        combine_bwd_kernel<__nv_bfloat16><<<blocks, 256, 0, s>>>(
-            (const __nv_bfloat16*)dout, (const __nv_bfloat16*)y_perm, topk_w, slot_of, T, d, k,
-            (__nv_bfloat16*)dy_perm, dtopk_w);
-    else
-        combine_bwd_kernel<float><<<blocks, 256, 0, s>>>((const float*)dout, (const float*)y_perm,
-                                                         topk_w, slot_of, T, d, k, (float*)dy_perm,
-                                                         dtopk_w);
+#define MOE_CB(TT, KM)                                                                           \
+    combine_bwd_kernel<TT, KM><<<blocks, 256, 0, s>>>((const TT*)dout, (const TT*)y_perm, topk_w, \
+                                                      slot_of, T, d, k, (TT*)dy_perm, dtopk_w)
+    if (bf16) {
+        if (k <= 2) MOE_CB(__nv_bfloat16, 2);
+        else if (k <= 4) MOE_CB(__nv_bfloat16, 4);
+        else MOE_CB(__nv_bfloat16, 8);
+    } else {
+        if (k <= 2) MOE_CB(float, 2);
+        else if (k <= 4) MOE_CB(float, 4);
+        else MOE_CB(float, 8);
+    }
+#undef MOE_CB
     return cudaGetLastError();
 }
 

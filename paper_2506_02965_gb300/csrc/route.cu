@@ -247,51 +247,48 @@ __device__ __forceinline__ bool chunk_of(int64_t ci, const int32_t* po, int P, i
     return false;
 }
 
-// dlogits, one thread per token (Alg. 7 backward with the picks held fixed).
-template <int EMAX>
+// dlogits, one warp per token (Alg. 7 backward with the picks held fixed); lane l
+// holds experts l and l + 32.
 __global__ void __launch_bounds__(256) dlogits_kernel(
     const float* __restrict__ probs, const int32_t* __restrict__ topk_idx,
     const float* __restrict__ topk_w, const float* __restrict__ dtopk_w,
     const float* __restrict__ aux_coef, const int32_t* __restrict__ po, int P, int64_t Tn, int E,
     int k, int normalize, float* dlogits) {
-    const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int lane = threadIdx.x & 31;
+    const int64_t t = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
     if (t >= Tn) return;
     const int party = party_of(po, P, t);
-    float pr[EMAX], dp[EMAX];
-#pragma unroll
-    for (int e = 0; e < EMAX; ++e) {
-        pr[e] = (e < E) ? probs[t * E + e] : 0.f;
-        dp[e] = (e < E && aux_coef) ? aux_coef[party * E + e] : 0.f;
-    }
-    float inner = 0.f, S = 0.f;
+    const int e0 = lane, e1 = lane + 32;
+    const float p0 = e0 < E ? probs[t * E + e0] : 0.f;
+    const float p1 = e1 < E ? probs[t * E + e1] : 0.f;
+    // lane j < k holds pick j
+    const int ej = lane < k ? topk_idx[t * k + lane] : -1;
+    const float gj0 = lane < k ? dtopk_w[t * k + lane] : 0.f;
+    const float wj = lane < k ? topk_w[t * k + lane] : 0.f;
+    float gj = gj0;
     if (normalize) {
-        for (int j = 0; j < k; ++j) {
-            const int e = topk_idx[t * k + j];
-            inner += dtopk_w[t * k + j] * topk_w[t * k + j];
-            if (e >= 0 && e < E) S += probs[t * E + e];
-        }
+        const float inner = warp_sum(gj0 * wj);
+        const float S = warp_sum((ej >= 0 && ej < E) ? probs[t * E + ej] : 0.f);
+        gj = (gj0 - inner) / S;
     }
+    float dp0 = (aux_coef && e0 < E) ? aux_coef[party * E + e0] : 0.f;
+    float dp1 = (aux_coef && e1 < E) ? aux_coef[party * E + e1] : 0.f;
     for (int j = 0; j < k; ++j) {
-        const int e = topk_idx[t * k + j];
-        float g = dtopk_w[t * k + j];
-        if (normalize) g = (g - inner) / S;
-#pragma unroll
-        for (int q = 0; q < EMAX; ++q)
-            if (q == e) dp[q] += g;
+        const int e = __shfl_sync(0xffffffffu, ej, j);
+        const float g = __shfl_sync(0xffffffffu, gj, j);
+        if (e == e0) dp0 += g;
+        if (e == e1) dp1 += g;
     }
-    float dot = 0.f;
-#pragma unroll
-    for (int e = 0; e < EMAX; ++e) dot = fmaf(dp[e], pr[e], dot);
-#pragma unroll
-    for (int e = 0; e < EMAX; ++e)
-        if (e < E) dlogits[t * E + e] = pr[e] * (dp[e] - dot);
+    const float dot = warp_sum(dp0 * p0 + dp1 * p1);
+    if (e0 < E) dlogits[t * E + e0] = p0 * (dp0 - dot);
+    if (e1 < E) dlogits[t * E + e1] = p1 * (dp1 - dot);
 }
 
 // Partial dW_r = dlogits^T x and db over one chunk of RB_CH tokens of one party, for
 // a tile of RB_ET experts and a column slab. The two thread halves take alternate
 // tokens of the chunk and are added in a fixed order at the end.
 constexpr int RB_CH = 32;   // tokens per chunk
-constexpr int RB_ET = 16;   // experts per tile
+constexpr int RB_ET = 8;    // experts per tile
 constexpr int RB_HALF = 128;  // threads per half
 
 template <typename T>
@@ -371,13 +368,17 @@ __global__ void __launch_bounds__(2 * RB_HALF) route_bwd_partial_kernel(
     }
 }
 
-// Sum the partials of each party's chunks in chunk order (four interleaved running
-// sums, combined in a fixed order).
+// Sum the partials of each party's chunks: a block takes 32 outputs; thread group g
+// (of 8) adds chunks g, g+8, ... in order, then group 0 adds the 8 group sums in order.
+constexpr int RR_OUT = 32, RR_GRP = 8;
+
 template <typename T>
-__global__ void __launch_bounds__(256) route_bwd_reduce_kernel(
+__global__ void __launch_bounds__(RR_OUT * RR_GRP) route_bwd_reduce_kernel(
     const float* __restrict__ part_dw, const float* __restrict__ part_db,
     const int32_t* __restrict__ po, int P, int64_t Tn, int d, int E, T* dw_router, float* dbias) {
-    const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    __shared__ float s_sum[RR_GRP][RR_OUT];
+    const int o = threadIdx.x % RR_OUT, g = threadIdx.x / RR_OUT;
+    const int64_t i = (int64_t)blockIdx.x * RR_OUT + o;
     const int64_t per_party = (int64_t)E * d;
     auto crange = [&](int p, int64_t* first, int64_t* cnt) {
         int64_t base = 0;
@@ -388,24 +389,24 @@ __global__ void __launch_bounds__(256) route_bwd_reduce_kernel(
             base += nc;
         }
     };
-    if (i < (int64_t)P * per_party) {
+    float acc = 0.f;
+    const bool ok = i < (int64_t)P * per_party;
+    if (ok) {
         const int p = (int)(i / per_party);
         const int64_t rem = i % per_party;
         int64_t first, cnt;
         crange(p, &first, &cnt);
-        const float* src = part_dw + first * per_party + rem;
-        float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
-        int64_t c = 0;
-        for (; c + 3 < cnt; c += 4) {
-            s0 += src[c * per_party];
-            s1 += src[(c + 1) * per_party];
-            s2 += src[(c + 2) * per_party];
-            s3 += src[(c + 3) * per_party];
-        }
-        for (; c < cnt; ++c) s0 += src[c * per_party];
-        Elem<T>::store(dw_router + i, (s0 + s1) + (s2 + s3));
+        for (int64_t c = g; c < cnt; c += RR_GRP) acc += part_dw[(first + c) * per_party + rem];
     }
-    if (dbias && i < (int64_t)P * E) {
+    s_sum[g][o] = acc;
+    __syncthreads();
+    if (g == 0 && ok) {
+        float tot = 0.f;
+#pragma unroll
+        for (int q = 0; q < RR_GRP; ++q) tot += s_sum[q][o];
+        Elem<T>::store(dw_router + i, tot);
+    }
+    if (dbias && g == 0 && i < (int64_t)P * E) {
         const int p = (int)(i / E), e = (int)(i % E);
         int64_t first, cnt;
         crange(p, &first, &cnt);
@@ -481,16 +482,9 @@ static cudaError_t launch_route_bwd_t(const RouteBwdArgs& a, void* ws, cudaStrea
     float* part_dw = (float*)ws;
     float* part_db = part_dw + nch * a.E * a.d;
     if (a.T > 0) {
-        const unsigned blocks = (unsigned)((a.T + 63) / 64);
-#define MOE_DZ(EM)                                                                             \
-    dlogits_kernel<EM><<<blocks, 64, 0, s>>>(a.probs, a.topk_idx, a.topk_w, a.dtopk_w,        \
-                                              a.aux_coef, a.po, a.P, a.T, a.E, a.k,            \
-                                              a.normalize, a.dlogits)
-        if (a.E <= 8) MOE_DZ(8);
-        else if (a.E <= 16) MOE_DZ(16);
-        else if (a.E <= 32) MOE_DZ(32);
-        else MOE_DZ(64);
-#undef MOE_DZ
+        const unsigned blocks = (unsigned)((a.T + 7) / 8);
+        dlogits_kernel<<<blocks, 256, 0, s>>>(a.probs, a.topk_idx, a.topk_w, a.dtopk_w, a.aux_coef,
+                                              a.po, a.P, a.T, a.E, a.k, a.normalize, a.dlogits);
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
     }
@@ -509,7 +503,7 @@ static cudaError_t launch_route_bwd_t(const RouteBwdArgs& a, void* ws, cudaStrea
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     const int64_t total = (int64_t)a.P * a.E * a.d;
-    route_bwd_reduce_kernel<T><<<(unsigned)((total + 255) / 256), 256, 0, s>>>(
+    route_bwd_reduce_kernel<T><<<(unsigned)((total + RR_OUT - 1) / RR_OUT), RR_OUT * RR_GRP, 0, s>>>(
         part_dw, part_db, a.po, a.P, a.T, a.d, a.E, (T*)a.dw_router, a.dbias);
     return cudaGetLastError();
 }
