@@ -28,7 +28,12 @@ constexpr int EPI_WARPS = 4;
 constexpr int THREADS = 64 + 32 * EPI_WARPS;  // TMA warp, MMA warp, epilogue warps
 constexpr int EPI_BOX = 32;                     // TMA-store box: 32 columns x 32 rows (bf16)
 constexpr int EPI_BUF_BYTES = EPI_BOX * EPI_BOX * 2;
-constexpr int EPI_STAGE_BYTES = 3 * EPI_BUF_BYTES;  // per epilogue warp: up to 3 outputs
+// per epilogue warp: up to 3 output boxes, or for the SwiGLU backward 2 x (G, U) boxes
+constexpr int EPI_STAGE_BYTES = 3 * EPI_BUF_BYTES;
+constexpr int EPI_STAGE_BYTES_BWD = 4 * EPI_BUF_BYTES;
+__host__ __device__ constexpr int epi_stage_bytes(int epi) {
+    return epi == EPI_SWIGLU_BWD ? EPI_STAGE_BYTES_BWD : EPI_STAGE_BYTES;
+}
 constexpr int MAX_GROUPS = 128;
 
 struct Params {
@@ -328,7 +333,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     constexpr int TMEM_COLS = (2 * BN <= 32) ? 32 : (2 * BN <= 64) ? 64 : (2 * BN <= 128) ? 128 : (2 * BN <= 256) ? 256 : 512;
 
     extern __shared__ uint8_t smem_raw[];
-    __shared__ uint64_t bars[2 * STAGES + 5];
+    __shared__ uint64_t bars[2 * STAGES + 5 + 2 * EPI_WARPS];
     __shared__ uint32_t s_tmem;
     __shared__ int s_abort;
     __shared__ int s_tile_start[MAX_GROUPS + 1];
@@ -422,6 +427,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             mbar_init(tempty_bar(a), 32 * EPI_WARPS);
         }
         mbar_init(drain_bar, 1);
+        for (int i = 0; i < 2 * EPI_WARPS; ++i) mbar_init(bar0 + 8u * (2 * STAGES + 5 + i), 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     if (warp == 1) {
@@ -584,10 +590,34 @@ __global__ void __launch_bounds__(THREADS, 1)
         // group's last row (the last M tile of an expert) is written row by row instead.
         const int q = warp & 3;
         const int row_local = q * 32 + lane;
-        uint8_t* stg = stage_out + (size_t)(warp - 2) * EPI_STAGE_BYTES;
+        uint8_t* stg = stage_out + (size_t)(warp - 2) * epi_stage_bytes(EPI);
         const uint32_t stg_u32 = smem_u32(stg);
         int acc = 0;
         uint32_t acc_phase = 0;
+        // SwiGLU backward: TMA loads of G/U chunk boxes into two staging buffers
+        const uint32_t gu_bar0 = bar0 + 8u * (2 * STAGES + 5 + 2 * (warp - 2));
+        uint32_t gu_issued = 0;  // chunks whose loads were issued (this warp)
+        uint32_t gu_chunk = 0;   // chunks consumed
+        auto gu_issue = [&](const Tile& tn, int cn) {
+            if constexpr (EPI == EPI_SWIGLU_BWD) {
+                const int b = gu_issued & 1;
+                if (lane == 0) {
+                    bulk_wait_read0();  // earlier stores out of this buffer have read it
+                    const uint32_t dst = stg_u32 + (2 * b) * EPI_BUF_BYTES;
+                    const int row0 = (int)(tn.out_row + tn.m0 + q * 32);
+                    mbar_expect_tx(gu_bar0 + 8u * b, 2 * EPI_BUF_BYTES);
+                    tma_load_2d(dst, &tmO1, gu_bar0 + 8u * b, tn.n0 + 32 * cn, row0);
+                    tma_load_2d(dst + EPI_BUF_BYTES, &tmO1, gu_bar0 + 8u * b, p.F + tn.n0 + 32 * cn, row0);
+                }
+                ++gu_issued;
+            }
+        };
+        auto gu_wait = [&](int b, uint32_t parity) -> bool {
+            return mbar_wait(gu_bar0 + 8u * b, parity, abort_flag, limit);
+        };
+        if constexpr (EPI == EPI_SWIGLU_BWD) {
+            if ((int)blockIdx.x < total_tiles) gu_issue(tile_at(blockIdx.x), 0);
+        }
         for (int t = blockIdx.x; t < total_tiles; t += gridDim.x) {
             const Tile ti = tile_at(t);
             const int m = ti.m0 + row_local;
@@ -616,37 +646,32 @@ __global__ void __launch_bounds__(THREADS, 1)
                 }
             };
             if constexpr (EPI == EPI_SWIGLU_BWD) {
-                // dA in TMEM; G and U come from h_gu. The next chunk's loads are in flight
-                // while the current one is computed; the first are issued before the wait.
+                // dA in TMEM. G and U of each 32-column chunk arrive by TMA in one of two
+                // staging buffers (the next chunk's load is in flight while this one is
+                // computed); dG and dU overwrite them in place and leave by TMA store.
                 const int F = p.F;
-                const __nv_bfloat16* __restrict__ hgu =
-                    (const __nv_bfloat16*)p.aux + (ti.out_row + m) * (int64_t)(2 * F) + ti.n0;
                 __nv_bfloat16* dh = (__nv_bfloat16*)p.out0 + (ti.out_row + m) * (int64_t)(2 * F) + ti.n0;
-                uint4 gc[4], uc[4];
-#pragma unroll
-                for (int v = 0; v < 4; ++v) {
-                    gc[v] = valid ? ldg_nc(hgu + 8 * v) : make_uint4(0, 0, 0, 0);
-                    uc[v] = valid ? ldg_nc(hgu + F + 8 * v) : make_uint4(0, 0, 0, 0);
-                }
+                constexpr int NCH = BN / 32;
                 if (!mbar_wait(tfull_bar(acc), acc_phase, abort_flag, limit)) break;
                 fence_after();
+                bool stop = false;
 #pragma unroll 1
-                for (int c = 0; c < BN / 32; ++c) {
-                    uint4 gn[4], un[4];
-                    if (c + 1 < BN / 32) {
-#pragma unroll
-                        for (int v = 0; v < 4; ++v) {
-                            gn[v] = valid ? ldg_nc(hgu + 32 * (c + 1) + 8 * v) : make_uint4(0, 0, 0, 0);
-                            un[v] = valid ? ldg_nc(hgu + F + 32 * (c + 1) + 8 * v) : make_uint4(0, 0, 0, 0);
-                        }
-                    }
+                for (int c = 0; c < NCH; ++c) {
+                    // prefetch the next chunk (of this tile, or the first of the next tile)
+                    if (c + 1 < NCH) gu_issue(ti, c + 1);
+                    else if (t + (int)gridDim.x < total_tiles) gu_issue(tile_at(t + gridDim.x), 0);
+                    const int b = gu_chunk & 1;
+                    if (!gu_wait(b, (gu_chunk >> 1) & 1)) { stop = true; break; }
+                    uint8_t* gbuf = stg + (2 * b) * EPI_BUF_BYTES + lane * 64;
+                    uint8_t* ubuf = gbuf + EPI_BUF_BYTES;
                     float da[32], dG[32], dU[32];
                     tmem_ld32(tbase + 32 * c, da);
 #pragma unroll
                     for (int v = 0; v < 4; ++v) {
+                        const int sw = (v ^ ((lane >> 1) & 3)) << 4;
                         float G[8], U[8];
-                        unpack8(gc[v], G);
-                        unpack8(uc[v], U);
+                        unpack8(*reinterpret_cast<const uint4*>(gbuf + sw), G);
+                        unpack8(*reinterpret_cast<const uint4*>(ubuf + sw), U);
 #pragma unroll
                         for (int i = 0; i < 8; ++i) {
                             const float sg = __fdividef(1.0f, 1.0f + __expf(-G[i]));
@@ -655,19 +680,25 @@ __global__ void __launch_bounds__(THREADS, 1)
                             dG[8 * v + i] = d * U[i] * sg * (1.0f + G[i] * (1.0f - sg));
                         }
                     }
-                    const float* vals[2] = {dG, dU};
-                    const CUtensorMap* maps[2] = {&tmO0, &tmO0};
-                    const int cols[2] = {ti.n0 + 32 * c, F + ti.n0 + 32 * c};
-                    __nv_bfloat16* direct[2] = {dh + 32 * c, dh + F + 32 * c};
-                    emit(2, vals, maps, cols, direct);
-                    if (c + 1 < BN / 32) {
-#pragma unroll
-                        for (int v = 0; v < 4; ++v) {
-                            gc[v] = gn[v];
-                            uc[v] = un[v];
+                    if (full_box) {
+                        store_row32_sw64(gbuf, lane, dG);
+                        store_row32_sw64(ubuf, lane, dU);
+                        fence_proxy_async();
+                        __syncwarp();
+                        if (lane == 0) {
+                            const uint32_t src = stg_u32 + (2 * b) * EPI_BUF_BYTES;
+                            tma_store_2d(&tmO0, src, ti.n0 + 32 * c, (int)grow0);
+                            tma_store_2d(&tmO0, src + EPI_BUF_BYTES, F + ti.n0 + 32 * c, (int)grow0);
+                            bulk_commit();
                         }
+                    } else if (valid) {
+                        store_row32(dh + 32 * c, dG);
+                        store_row32(dh + F + 32 * c, dU);
                     }
+                    __syncwarp();
+                    ++gu_chunk;
                 }
+                if (stop) break;
             } else {
                 if (!mbar_wait(tfull_bar(acc), acc_phase, abort_flag, limit)) break;
                 fence_after();
@@ -723,6 +754,14 @@ __global__ void __launch_bounds__(THREADS, 1)
             }
         }
         if (lane == 0) bulk_wait0();  // every TMA store of this warp has completed
+        if constexpr (EPI == EPI_SWIGLU_BWD) {
+            // loads issued but not consumed (only after an abort): let them land
+            for (uint32_t c = gu_chunk; c < gu_issued; ++c) {
+                const uint64_t t0 = gtimer();
+                while (!mbar_try(gu_bar0 + 8u * (c & 1), (c >> 1) & 1) && gtimer() - t0 < limit) {
+                }
+            }
+        }
     }
     fence_before();
     __syncthreads();
@@ -792,8 +831,8 @@ static cudaError_t launch(const CUtensorMap& ma, const CUtensorMap& mb, const CU
                           const CUtensorMap& mo1, const Params& p, int64_t tiles_ub,
                           cudaStream_t s) {
     auto kern = grouped_gemm_kernel<BN, B_MN, VAR_K, EPI>;
-    const int extra_max = EPI == EPI_ROUTE ? 64 * 64 * 4 : EPI_WARPS * EPI_STAGE_BYTES;
-    const int extra = EPI == EPI_ROUTE ? p.hist_n * 4 : EPI_WARPS * EPI_STAGE_BYTES;
+    const int extra_max = EPI == EPI_ROUTE ? 64 * 64 * 4 : EPI_WARPS * epi_stage_bytes(EPI);
+    const int extra = EPI == EPI_ROUTE ? p.hist_n * 4 : EPI_WARPS * epi_stage_bytes(EPI);
     const int smem_max = STAGES * (BM * BK * 2 + BN * BK * 2) + 1024 + extra_max;
     const int smem = STAGES * (BM * BK * 2 + BN * BK * 2) + 1024 + extra;
     static bool attr_set = false;
@@ -865,8 +904,9 @@ cudaError_t launch_gemm_m(const GemmMArgs& g, bool bf16, cudaStream_t s) {
     if (g.epi == EPI_SWIGLU_BWD) {
         p.F = g.N;
         if (!make_map(&mo0, g.out0, 2 * (int64_t)g.N, o_rows, 0, true)) return cudaErrorInvalidValue;
-        if (g.N % 256 == 0) return launch<256, true, false, EPI_SWIGLU_BWD>(ma, mb, mo0, mo0, p, mt_ub * (g.N / 256), s);
-        return launch<128, true, false, EPI_SWIGLU_BWD>(ma, mb, mo0, mo0, p, mt_ub * (g.N / 128), s);
+        if (!make_map(&mo1, g.aux, 2 * (int64_t)g.N, o_rows, 0, true)) return cudaErrorInvalidValue;
+        if (g.N % 256 == 0) return launch<256, true, false, EPI_SWIGLU_BWD>(ma, mb, mo0, mo1, p, mt_ub * (g.N / 256), s);
+        return launch<128, true, false, EPI_SWIGLU_BWD>(ma, mb, mo0, mo1, p, mt_ub * (g.N / 128), s);
     }
     if (!make_map(&mo0, g.out0, g.N, o_rows, 0, true)) return cudaErrorInvalidValue;
     if (g.N % 256 == 0) return launch<256, true, false, EPI_STORE>(ma, mb, mo0, mo0, p, mt_ub * (g.N / 256), s);
