@@ -4,6 +4,7 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
+#include <mutex>
 #include <string>
 
 #include "../../include/moe.h"
@@ -84,6 +85,36 @@ moe_status check_parties(const moe_config* c, const int32_t* po) {
 }
 
 size_t elem_size(const moe_config* c) { return c->dtype == MOE_BF16 ? 2 : 4; }
+
+// A second stream per device on which the backward runs the weight-gradient GEMMs
+// while the input-gradient GEMMs run on the caller's stream, so that the tail wave of
+// one persistent kernel is filled by the other. Fork and join are event waits, so all
+// work stays ordered with respect to the caller's stream. Created on the first call
+// on a device (that call must not be inside a stream capture).
+struct SideStream {
+    cudaStream_t s = nullptr;
+    cudaEvent_t fork = nullptr, mid = nullptr, join = nullptr;
+};
+constexpr int kMaxDev = 64;
+SideStream g_side[kMaxDev];
+std::mutex g_side_mu;
+
+cudaError_t side_stream(SideStream** out) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDev) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lk(g_side_mu);
+    SideStream& ss = g_side[dev];
+    if (!ss.s) {
+        if ((e = cudaStreamCreateWithFlags(&ss.s, cudaStreamNonBlocking)) != cudaSuccess) return e;
+        if ((e = cudaEventCreateWithFlags(&ss.fork, cudaEventDisableTiming)) != cudaSuccess) return e;
+        if ((e = cudaEventCreateWithFlags(&ss.mid, cudaEventDisableTiming)) != cudaSuccess) return e;
+        if ((e = cudaEventCreateWithFlags(&ss.join, cudaEventDisableTiming)) != cudaSuccess) return e;
+    }
+    *out = &ss;
+    return cudaSuccess;
+}
 
 }  // namespace
 
@@ -424,7 +455,6 @@ moe_status moe_expert_ffn_bwd(const moe_config* cfg, const void* x_perm, const i
     a.epi = EPI_SWIGLU_BWD;
     a.aux = h_gu;
     a.out0 = dh;
-    if ((st = cuda_status(launch_gemm_m(a, bf16, s), "expert dA gemm"))) return st;
     // dXp = dH W1
     GemmMArgs b{};
     b.G = E;
@@ -437,7 +467,6 @@ moe_status moe_expert_ffn_bwd(const moe_config* cfg, const void* x_perm, const i
     b.K = 2 * F;
     b.epi = EPI_STORE;
     b.out0 = dx_perm;
-    if ((st = cuda_status(launch_gemm_m(b, bf16, s), "expert dX gemm"))) return st;
     // dW2[e] = dY_e^T A_e ; dW1[e] = dH_e^T Xp_e
     GemmKArgs w2g{};
     w2g.G = E;
@@ -447,7 +476,6 @@ moe_status moe_expert_ffn_bwd(const moe_config* cfg, const void* x_perm, const i
     w2g.M = d;
     w2g.N = F;
     w2g.out = dw2;
-    if ((st = cuda_status(launch_gemm_k(w2g, bf16, s), "expert dW2 gemm"))) return st;
     GemmKArgs w1g{};
     w1g.G = E;
     w1g.rows = GroupRows{offsets, (int)TK, 0, 0, 0};
@@ -456,7 +484,20 @@ moe_status moe_expert_ffn_bwd(const moe_config* cfg, const void* x_perm, const i
     w1g.M = 2 * F;
     w1g.N = d;
     w1g.out = dw1;
-    if ((st = cuda_status(launch_gemm_k(w1g, bf16, s), "expert dW1 gemm"))) return st;
+    // caller stream: dA then dX; side stream: dW2 (needs only dY and A) alongside dA,
+    // then dW1 once dH exists
+    SideStream* ss = nullptr;
+    if ((st = cuda_status(side_stream(&ss), "side stream"))) return st;
+    if ((st = cuda_status(cudaEventRecord(ss->fork, s), "fork"))) return st;
+    if ((st = cuda_status(cudaStreamWaitEvent(ss->s, ss->fork, 0), "fork"))) return st;
+    if ((st = cuda_status(launch_gemm_k(w2g, bf16, ss->s), "expert dW2 gemm"))) return st;
+    if ((st = cuda_status(launch_gemm_m(a, bf16, s), "expert dA gemm"))) return st;
+    if ((st = cuda_status(cudaEventRecord(ss->mid, s), "mid"))) return st;
+    if ((st = cuda_status(launch_gemm_m(b, bf16, s), "expert dX gemm"))) return st;
+    if ((st = cuda_status(cudaStreamWaitEvent(ss->s, ss->mid, 0), "mid"))) return st;
+    if ((st = cuda_status(launch_gemm_k(w1g, bf16, ss->s), "expert dW1 gemm"))) return st;
+    if ((st = cuda_status(cudaEventRecord(ss->join, ss->s), "join"))) return st;
+    if ((st = cuda_status(cudaStreamWaitEvent(s, ss->join, 0), "join"))) return st;
     if (S) {
         GemmMArgs sa = a;
         sa.G = S;

@@ -66,6 +66,8 @@ class MoELayer:
         self.dw_router = z(P, E, d)
         self.dbias = z(P, E, dtype=f32)
         self.dx = z(T, d)
+        # the router backward runs beside the expert backward on this stream
+        self.side = torch.cuda.Stream(device=device)
         self.ws_bytes = L.moe_workspace_size(self.cfg)
         self.workspace = torch.empty(max(self.ws_bytes, 16), dtype=torch.uint8, device=device)
 
@@ -114,20 +116,28 @@ class MoELayer:
     def backward(self, stream=None, with_aux: bool = True, mark=None):
         c = self.cfg
         mark = mark or (lambda name: None)
+        main = stream if stream is not None else torch.cuda.current_stream()
         L.moe_combine_bwd(c, self.dout, self.y_perm, self.topk_w, self.slot_of, self.dy_perm,
-                          self.dtopk_w, stream=stream)
+                          self.dtopk_w, stream=main)
+        # the router backward needs only the gate gradients: run it beside the experts
+        fork = torch.cuda.Event()
+        fork.record(main)
+        self.side.wait_event(fork)
+        L.moe_route_bwd(c, self.x, self.w_router, self.probs, self.topk_idx, self.topk_w,
+                        self.dtopk_w, self.aux_coef if with_aux else None, self._po(),
+                        self.dlogits, self.dw_router, self.dbias, self.workspace, self.ws_bytes,
+                        stream=self.side)
+        join = torch.cuda.Event()
+        join.record(self.side)
         mark("ffn_bwd_begin")
         L.moe_expert_ffn_bwd(c, self.x_perm, self.offsets, self.w1, self.w2, self.h_gu, self.act,
                              self.dy_perm, self.dh, self.dx_perm, self.dw1, self.dw2, self.x,
                              self.dout, self.ws1, self.ws2, self.h_gu_sh, self.act_sh, self.dh_sh,
-                             self.dx_sh, self.dws1, self.dws2, stream=stream)
+                             self.dx_sh, self.dws1, self.dws2, stream=main)
         mark("ffn_bwd_end")
-        L.moe_route_bwd(c, self.x, self.w_router, self.probs, self.topk_idx, self.topk_w,
-                        self.dtopk_w, self.aux_coef if with_aux else None, self._po(),
-                        self.dlogits, self.dw_router, self.dbias, self.workspace, self.ws_bytes,
-                        stream=stream)
+        main.wait_event(join)
         L.moe_dispatch_bwd(c, self.dx_perm, self.slot_of, self.dlogits, self.w_router, self._po(),
-                           self.dx_sh, self.dx, stream=stream)
+                           self.dx_sh, self.dx, stream=main)
 
     def step(self, stream=None, mark=None):
         """One fwd+bwd pass of the whole layer. ``mark(name)`` (optional) is called at
