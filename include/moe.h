@@ -237,6 +237,13 @@ moe_status moe_device_status(moe_stream_t stream, int32_t* code /* HOST out */);
  * (default 2e9). A wait that runs out records MOE_ERR_TIMEOUT and the kernel returns. */
 moe_status moe_set_wait_limit_ns(uint64_t ns);
 
+/* Tile shape of the 256-wide expert GEMMs whose rows vary per expert (forward, dA,
+ * dX). on = 0 (default): one CTA per 128 x 256 tile; on = 1: a pair of CTAs on two SMs
+ * computes each 256 x 256 tile with tcgen05 cta_group::2 MMAs, each SM holding half of
+ * the B operand (measured slower than on = 0 on GB300 for these shapes). Results agree
+ * up to fp32 summation order. */
+moe_status moe_set_gemm_pairs(int on);
+
 const char* moe_status_string(moe_status s);
 /* Reason for the last MOE_ERR_INVALID_ARG / MOE_ERR_CUDA returned on this thread. */
 const char* moe_last_error(void);

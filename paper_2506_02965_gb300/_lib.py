@@ -74,6 +74,7 @@ _SIGS = {
     "moe_dispatch_bwd": [_CFG] + [P] * 8,
     "moe_device_status": [P, ctypes.POINTER(ctypes.c_int32)],
     "moe_set_wait_limit_ns": [ctypes.c_uint64],
+    "moe_set_gemm_pairs": [ctypes.c_int],
 }
 for _n, _a in _SIGS.items():
     f = getattr(_lib, _n)
@@ -146,6 +147,10 @@ def moe_workspace_size(cfg) -> int:
 
 def moe_set_wait_limit_ns(ns: int):
     _check(_lib.moe_set_wait_limit_ns(int(ns)), "moe_set_wait_limit_ns")
+
+
+def moe_set_gemm_pairs(on: int):
+    _check(_lib.moe_set_gemm_pairs(int(on)), "moe_set_gemm_pairs")
 
 
 def moe_device_status(stream=None) -> int:

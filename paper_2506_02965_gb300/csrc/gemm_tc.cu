@@ -105,6 +105,71 @@ __device__ __noinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile i
         }
     }
 }
+// --- CTA-pair (cta_group::2) helpers
+__device__ __forceinline__ uint32_t cluster_rank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+// shared::cluster address of the same shared-memory offset in CTA `rank` of the cluster
+__device__ __forceinline__ uint32_t map_to_rank(uint32_t addr, uint32_t rank) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+    return r;
+}
+__device__ __forceinline__ void mbar_expect_tx_remote(uint32_t cluster_bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.release.cluster.shared::cluster.b64 _, [%0], %1;" ::"r"(
+                     cluster_bar),
+                 "r"(bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_bar) {
+    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_bar)
+                 : "memory");
+}
+__device__ __forceinline__ bool mbar_try_cluster(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+// TMA load into this CTA's shared memory whose completion is counted on a barrier
+// that may live in the peer CTA of the pair (the leader's "full" barrier)
+__device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap* map,
+                                                 uint32_t cluster_bar, int c0, int c1) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes "
+        "[%0], [%1, {%3, %4}], [%2];" ::"r"(dst),
+        "l"((uint64_t)map), "r"(cluster_bar), "r"(c0), "r"(c1)
+        : "memory");
+}
+__device__ __forceinline__ void mma_bf16_pair(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
+                                              uint32_t idesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+// commit the pair's MMAs to the barrier at this offset in every CTA of `mask`
+__device__ __forceinline__ void mma_commit_pair(uint32_t bar, uint16_t mask) {
+    asm volatile(
+        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 "
+        "[%0], %1;" ::"r"(bar),
+        "h"(mask)
+        : "memory");
+}
+__device__ __forceinline__ void cluster_sync_all() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::
+                     : "memory");
+}
+
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, uint32_t bar,
                                             int c0, int c1) {
     asm volatile(
@@ -224,10 +289,10 @@ __device__ __forceinline__ uint64_t smem_desc(uint32_t saddr, uint32_t lbo, uint
 }
 // Instruction descriptor of kind::f16: fp32 D [4,6), bf16 A [7,10), bf16 B [10,13),
 // A major [15], B major [16] (1 = MN-major), N>>3 [17,23), M>>4 [24,29).
-template <int BN, bool A_MN, bool B_MN>
+template <int BN, bool A_MN, bool B_MN, int M = BM>
 __host__ __device__ constexpr uint32_t instr_desc() {
     return (1u << 4) | (1u << 7) | (1u << 10) | ((A_MN ? 1u : 0u) << 15) |
-           ((B_MN ? 1u : 0u) << 16) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
+           ((B_MN ? 1u : 0u) << 16) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
 }
 
 // ------------------------------------------------------------------------ tile geometry
@@ -319,27 +384,36 @@ __device__ __forceinline__ void route_epilogue(const Params& p, const Tile& ti, 
 }
 
 // ------------------------------------------------------------------------ the kernel
-template <int BN, bool B_MN, bool VAR_K, int EPI>
+// PAIR: the two CTAs of a cluster compute one 256 x BN tile with tcgen05 cta_group::2
+// MMAs issued by CTA 0: each CTA holds 128 rows of A and BN/2 rows of B in its own
+// shared memory and 128 rows of the accumulator in its own TMEM.
+template <int BN, bool B_MN, bool VAR_K, int EPI, bool PAIR = false>
 __global__ void __launch_bounds__(THREADS, 1)
     grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA,
                         const __grid_constant__ CUtensorMap tmB,
                         const __grid_constant__ CUtensorMap tmO0,
                         const __grid_constant__ CUtensorMap tmO1, const Params p) {
     constexpr bool A_MN = VAR_K;
+    constexpr int NPAIR = PAIR ? 2 : 1;
+    constexpr int BNL = BN / NPAIR;  // B rows held by this CTA
+    constexpr int BMP = BM * NPAIR;  // rows of one (pair) tile
+    constexpr int NST = PAIR ? 6 : STAGES;
     constexpr uint32_t A_BYTES = BM * BK * 2;
-    constexpr uint32_t B_BYTES = BN * BK * 2;
+    constexpr uint32_t B_BYTES = BNL * BK * 2;
     constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
-    constexpr uint32_t IDESC = instr_desc<BN, A_MN, B_MN>();
+    constexpr uint32_t IDESC = instr_desc<BN, A_MN, B_MN, BMP>();
     constexpr int TMEM_COLS = (2 * BN <= 32) ? 32 : (2 * BN <= 64) ? 64 : (2 * BN <= 128) ? 128 : (2 * BN <= 256) ? 256 : 512;
 
     extern __shared__ uint8_t smem_raw[];
-    __shared__ uint64_t bars[2 * STAGES + 5 + 2 * EPI_WARPS];
+    __shared__ uint64_t bars[2 * NST + 5 + 2 * EPI_WARPS];
     __shared__ uint32_t s_tmem;
     __shared__ int s_abort;
     __shared__ int s_tile_start[MAX_GROUPS + 1];
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     volatile int* abort_flag = &s_abort;
+    const uint32_t rank = PAIR ? cluster_rank() : 0u;
+    const int tile0 = (int)blockIdx.x / NPAIR, tile_step = (int)gridDim.x / NPAIR;
 
     // group -> tile prefix
     const int tiles_n = (EPI == EPI_SWIGLU_FWD) ? p.N / 256 : (EPI == EPI_ROUTE) ? 1 : p.N / BN;
@@ -349,10 +423,10 @@ __global__ void __launch_bounds__(THREADS, 1)
             s_tile_start[g] = acc;
             int mt;
             if (VAR_K) {
-                mt = p.Mout / BM;
+                mt = p.Mout / BMP;
             } else {
                 const int rows = p.offsets ? (p.offsets[g + 1] - p.offsets[g]) : p.rows;
-                mt = rows > 0 ? (rows + BM - 1) / BM : 0;
+                mt = rows > 0 ? (rows + BMP - 1) / BMP : 0;
             }
             acc += mt * tiles_n;
         }
@@ -361,7 +435,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
     __syncthreads();
     const int total_tiles = s_tile_start[p.G];
-    if ((int)blockIdx.x >= total_tiles) return;
+    if (tile0 >= total_tiles) return;  // uniform across the pair
 
     auto tile_at = [&](int t) -> Tile {
         Tile ti;
@@ -370,7 +444,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         const int local = t - s_tile_start[g];
         const int mt = local / tiles_n, nt = local % tiles_n;
         ti.g = g;
-        ti.m0 = mt * BM;
+        ti.m0 = mt * BMP + (int)rank * BM;
         ti.n0 = nt * ((EPI == EPI_SWIGLU_FWD) ? 128 : BN);
         int64_t r0, nrows, a0, b0, o0;
         if (p.offsets) {
@@ -405,40 +479,69 @@ __global__ void __launch_bounds__(THREADS, 1)
     const uint32_t raw_u32 = smem_u32(smem_raw);
     const uint32_t ring = raw_u32 + ((1024u - (raw_u32 & 1023u)) & 1023u);
     uint8_t* ring_ptr = smem_raw + (ring - raw_u32);
-    uint8_t* stage_out = ring_ptr + (size_t)STAGES * STAGE_BYTES;  // EPI_WARPS x EPI_STAGE_BYTES
+    uint8_t* stage_out = ring_ptr + (size_t)NST * STAGE_BYTES;  // EPI_WARPS x EPI_STAGE_BYTES
     int* route_hist = reinterpret_cast<int*>(stage_out);             // EPI_ROUTE has no staging
     if constexpr (EPI == EPI_ROUTE) {
         for (int i = threadIdx.x; i < p.hist_n; i += blockDim.x) route_hist[i] = 0;
     }
     const uint32_t bar0 = smem_u32(&bars[0]);
     auto full_bar = [&](int s) { return bar0 + 8u * s; };
-    auto empty_bar = [&](int s) { return bar0 + 8u * (STAGES + s); };
-    auto tfull_bar = [&](int a) { return bar0 + 8u * (2 * STAGES + a); };
-    auto tempty_bar = [&](int a) { return bar0 + 8u * (2 * STAGES + 2 + a); };
-    const uint32_t drain_bar = bar0 + 8u * (2 * STAGES + 4);
+    auto empty_bar = [&](int s) { return bar0 + 8u * (NST + s); };
+    auto tfull_bar = [&](int a) { return bar0 + 8u * (2 * NST + a); };
+    auto tempty_bar = [&](int a) { return bar0 + 8u * (2 * NST + 2 + a); };
+    const uint32_t drain_bar = bar0 + 8u * (2 * NST + 4);
+    // waits: cluster-scope acquire when the barrier also collects the peer's arrivals
+    auto wait_bar = [&](uint32_t bar, uint32_t parity) -> bool {
+        if constexpr (PAIR) {
+            if (mbar_try_cluster(bar, parity)) return true;
+            const uint64_t t0 = gtimer();
+            for (uint32_t it = 1;; ++it) {
+                if (mbar_try_cluster(bar, parity)) return true;
+                if ((it & 31u) == 0) {
+                    if (*abort_flag) return false;
+                    if (gtimer() - t0 > p.wait_ns) {
+                        *abort_flag = 1;
+                        record_status(MOE_ERR_TIMEOUT);
+                        return false;
+                    }
+                }
+            }
+        } else {
+            return mbar_wait(bar, parity, abort_flag, p.wait_ns);
+        }
+    };
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < STAGES; ++s) {
-            mbar_init(full_bar(s), 1);
+        for (int s = 0; s < NST; ++s) {
+            mbar_init(full_bar(s), NPAIR);  // one producer arrival per CTA of the pair
             mbar_init(empty_bar(s), 1);
         }
         for (int a = 0; a < 2; ++a) {
             mbar_init(tfull_bar(a), 1);
-            mbar_init(tempty_bar(a), 32 * EPI_WARPS);
+            mbar_init(tempty_bar(a), EPI_WARPS * NPAIR);  // one arrival per epilogue warp
         }
         mbar_init(drain_bar, 1);
-        for (int i = 0; i < 2 * EPI_WARPS; ++i) mbar_init(bar0 + 8u * (2 * STAGES + 5 + i), 1);
+        for (int i = 0; i < 2 * EPI_WARPS; ++i) mbar_init(bar0 + 8u * (2 * NST + 5 + i), 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     if (warp == 1) {
-        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
-                         smem_u32(&s_tmem)),
-                     "r"(TMEM_COLS)
-                     : "memory");
-        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+        if constexpr (PAIR) {
+            asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                             smem_u32(&s_tmem)),
+                         "r"(TMEM_COLS)
+                         : "memory");
+            asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+        } else {
+            asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                             smem_u32(&s_tmem)),
+                         "r"(TMEM_COLS)
+                         : "memory");
+            asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+        }
     }
     fence_before();
     __syncthreads();
+    if constexpr (PAIR) cluster_sync_all();  // the peer's barriers are initialised
     fence_after();
     const uint32_t tmem_base = s_tmem;
     const uint64_t limit = p.wait_ns;
@@ -448,50 +551,63 @@ __global__ void __launch_bounds__(THREADS, 1)
         if (lane == 0) {
             int stage = 0;
             uint32_t phase = 0;
-            int issued_phase[STAGES];
-            for (int s = 0; s < STAGES; ++s) issued_phase[s] = -1;
+            int issued_phase[NST];
+            for (int s = 0; s < NST; ++s) issued_phase[s] = -1;
             bool ok = true;
-            for (int t = blockIdx.x; t < total_tiles && ok; t += gridDim.x) {
+            // every TMA load is counted on the leader's full barrier (CTA 0 of a pair)
+            auto load = [&](uint32_t dst, const CUtensorMap* map, uint32_t fb, int c0, int c1) {
+                if constexpr (PAIR) tma_load_2d_pair(dst, map, fb, c0, c1);
+                else tma_load_2d(dst, map, fb, c0, c1);
+            };
+            for (int t = tile0; t < total_tiles && ok; t += tile_step) {
                 const Tile ti = tile_at(t);
                 for (int kb = 0; kb < ti.k_iters; ++kb) {
-                    if (!mbar_wait(empty_bar(stage), phase ^ 1u, abort_flag, limit)) {
+                    if (!wait_bar(empty_bar(stage), phase ^ 1u)) {
                         ok = false;
                         break;
                     }
                     const uint32_t sa = ring + stage * STAGE_BYTES;
                     const uint32_t sb = sa + A_BYTES;
-                    const uint32_t fb = full_bar(stage);
-                    mbar_expect_tx(fb, STAGE_BYTES);
+                    const uint32_t fb = PAIR ? map_to_rank(full_bar(stage), 0) : full_bar(stage);
+                    if constexpr (PAIR) mbar_expect_tx_remote(fb, STAGE_BYTES);
+                    else mbar_expect_tx(fb, STAGE_BYTES);
                     const int k0 = kb * BK;
                     if (!A_MN) {
-                        tma_load_2d(sa, &tmA, fb, k0, (int)(ti.a_row + ti.m0));
+                        load(sa, &tmA, fb, k0, (int)(ti.a_row + ti.m0));
                     } else {
 #pragma unroll
                         for (int i = 0; i < BM / 64; ++i)
-                            tma_load_2d(sa + i * 8192, &tmA, fb, ti.m0 + 64 * i, (int)(ti.a_row + k0));
+                            load(sa + i * 8192, &tmA, fb, ti.m0 + 64 * i, (int)(ti.a_row + k0));
                     }
                     if (EPI == EPI_SWIGLU_FWD) {
+                        // 128 gate rows then 128 up rows of the same features; in a pair the
+                        // leader holds the gate half and the peer the up half
                         const int64_t r = (int64_t)ti.g * p.b_group_rows + ti.n0;
-                        tma_load_2d(sb, &tmB, fb, k0, (int)r);
-                        tma_load_2d(sb + 128 * 128, &tmB, fb, k0, (int)(r + p.F));
+                        if constexpr (PAIR) {
+                            load(sb, &tmB, fb, k0, (int)(r + (rank ? p.F : 0)));
+                        } else {
+                            load(sb, &tmB, fb, k0, (int)r);
+                            load(sb + 128 * 128, &tmB, fb, k0, (int)(r + p.F));
+                        }
                     } else if (!B_MN) {
-                        tma_load_2d(sb, &tmB, fb, k0, (int)((int64_t)ti.g * p.b_group_rows + ti.n0));
+                        load(sb, &tmB, fb, k0, (int)((int64_t)ti.g * p.b_group_rows + ti.n0 + rank * BNL));
                     } else {
                         const int64_t krow = VAR_K ? (ti.b_row + k0) : ((int64_t)ti.g * p.b_group_rows + k0);
 #pragma unroll
-                        for (int i = 0; i < BN / 64; ++i)
-                            tma_load_2d(sb + i * 8192, &tmB, fb, ti.n0 + 64 * i, (int)krow);
+                        for (int i = 0; i < BNL / 64; ++i)
+                            load(sb + i * 8192, &tmB, fb, ti.n0 + (int)rank * BNL + 64 * i, (int)krow);
                     }
                     issued_phase[stage] = (int)phase;
-                    if (++stage == STAGES) {
+                    if (++stage == NST) {
                         stage = 0;
                         phase ^= 1u;
                     }
                 }
             }
-            if (!ok || *abort_flag) {
-                // let every copy this thread started land before the CTA exits
-                for (int s = 0; s < STAGES; ++s) {
+            if ((!ok || *abort_flag) && rank == 0) {
+                // let every copy started into this pair land before the CTAs exit (the
+                // leader's full barriers count the peer's bytes too)
+                for (int s = 0; s < NST; ++s) {
                     if (issued_phase[s] < 0) continue;
                     const uint64_t t0 = gtimer();
                     while (!mbar_try(full_bar(s), (uint32_t)issued_phase[s]) &&
@@ -508,16 +624,18 @@ __global__ void __launch_bounds__(THREADS, 1)
         uint32_t acc_phase = 0;
         bool ok = true;
         bool issued_any = false;
-        for (int t = blockIdx.x; t < total_tiles && ok; t += gridDim.x) {
+        // in a pair only the leader issues MMAs (they read both CTAs' shared memory and
+        // write both CTAs' TMEM)
+        for (int t = tile0; t < total_tiles && ok && rank == 0; t += tile_step) {
             const Tile ti = tile_at(t);
-            if (!mbar_wait(tempty_bar(acc), acc_phase ^ 1u, abort_flag, limit)) {
+            if (!wait_bar(tempty_bar(acc), acc_phase ^ 1u)) {
                 ok = false;
                 break;
             }
             fence_after();
             const uint32_t tmem_d = tmem_base + (uint32_t)(acc * BN);
             for (int kb = 0; kb < ti.k_iters; ++kb) {
-                if (!mbar_wait(full_bar(stage), phase, abort_flag, limit)) {
+                if (!wait_bar(full_bar(stage), phase)) {
                     ok = false;
                     break;
                 }
@@ -553,21 +671,27 @@ __global__ void __launch_bounds__(THREADS, 1)
                         else ad = smem_desc(sa + kk * 2048, 8192, 1024);
                         if (!B_MN) bd = smem_desc(sb + kk * 32, 16, 1024);
                         else bd = smem_desc(sb + kk * 2048, 8192, 1024);
-                        mma_bf16(tmem_d, ad, bd, IDESC, (kb | kk) ? 1u : 0u);
+                        if constexpr (PAIR) mma_bf16_pair(tmem_d, ad, bd, IDESC, (kb | kk) ? 1u : 0u);
+                        else mma_bf16(tmem_d, ad, bd, IDESC, (kb | kk) ? 1u : 0u);
                     }
-                    mma_commit(empty_bar(stage));
+                    if constexpr (PAIR) mma_commit_pair(empty_bar(stage), 3);  // both producers
+                    else mma_commit(empty_bar(stage));
                     issued_any = true;
                 }
                 __syncwarp();
-                if (++stage == STAGES) {
+                if (++stage == NST) {
                     stage = 0;
                     phase ^= 1u;
                 }
             }
             if (!ok) break;
             if (lane == 0) {
-                if (ti.k_iters > 0) mma_commit(tfull_bar(acc));
-                else mbar_arrive(tfull_bar(acc));
+                if constexpr (PAIR) {
+                    mma_commit_pair(tfull_bar(acc), 3);  // both CTAs' epilogues
+                } else {
+                    if (ti.k_iters > 0) mma_commit(tfull_bar(acc));
+                    else mbar_arrive(tfull_bar(acc));
+                }
             }
             __syncwarp();
             if (++acc == 2) {
@@ -577,7 +701,8 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
         if ((!ok || *abort_flag) && lane == 0 && issued_any) {
             // wait for every MMA this CTA issued before TMEM is released
-            mma_commit(drain_bar);
+            if constexpr (PAIR) mma_commit_pair(drain_bar, 1);
+            else mma_commit(drain_bar);
             const uint64_t t0 = gtimer();
             while (!mbar_try(drain_bar, 0) && gtimer() - t0 < limit) {
             }
@@ -595,7 +720,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         int acc = 0;
         uint32_t acc_phase = 0;
         // SwiGLU backward: TMA loads of G/U chunk boxes into two staging buffers
-        const uint32_t gu_bar0 = bar0 + 8u * (2 * STAGES + 5 + 2 * (warp - 2));
+        const uint32_t gu_bar0 = bar0 + 8u * (2 * NST + 5 + 2 * (warp - 2));
         uint32_t gu_issued = 0;  // chunks whose loads were issued (this warp)
         uint32_t gu_chunk = 0;   // chunks consumed
         auto gu_issue = [&](const Tile& tn, int cn) {
@@ -616,9 +741,9 @@ __global__ void __launch_bounds__(THREADS, 1)
             return mbar_wait(gu_bar0 + 8u * b, parity, abort_flag, limit);
         };
         if constexpr (EPI == EPI_SWIGLU_BWD) {
-            if ((int)blockIdx.x < total_tiles) gu_issue(tile_at(blockIdx.x), 0);
+            if (tile0 < total_tiles) gu_issue(tile_at(tile0), 0);
         }
-        for (int t = blockIdx.x; t < total_tiles; t += gridDim.x) {
+        for (int t = tile0; t < total_tiles; t += tile_step) {
             const Tile ti = tile_at(t);
             const int m = ti.m0 + row_local;
             const bool valid = m < ti.mvalid;
@@ -652,14 +777,14 @@ __global__ void __launch_bounds__(THREADS, 1)
                 const int F = p.F;
                 __nv_bfloat16* dh = (__nv_bfloat16*)p.out0 + (ti.out_row + m) * (int64_t)(2 * F) + ti.n0;
                 constexpr int NCH = BN / 32;
-                if (!mbar_wait(tfull_bar(acc), acc_phase, abort_flag, limit)) break;
+                if (!wait_bar(tfull_bar(acc), acc_phase)) break;
                 fence_after();
                 bool stop = false;
 #pragma unroll 1
                 for (int c = 0; c < NCH; ++c) {
                     // prefetch the next chunk (of this tile, or the first of the next tile)
                     if (c + 1 < NCH) gu_issue(ti, c + 1);
-                    else if (t + (int)gridDim.x < total_tiles) gu_issue(tile_at(t + gridDim.x), 0);
+                    else if (t + tile_step < total_tiles) gu_issue(tile_at(t + tile_step), 0);
                     const int b = gu_chunk & 1;
                     if (!gu_wait(b, (gu_chunk >> 1) & 1)) { stop = true; break; }
                     uint8_t* gbuf = stg + (2 * b) * EPI_BUF_BYTES + lane * 64;
@@ -700,7 +825,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                 }
                 if (stop) break;
             } else {
-                if (!mbar_wait(tfull_bar(acc), acc_phase, abort_flag, limit)) break;
+                if (!wait_bar(tfull_bar(acc), acc_phase)) break;
                 fence_after();
                 if constexpr (EPI == EPI_SWIGLU_FWD) {
                     // accumulator columns [0,128) = G, [128,256) = U of features n0 .. n0+127
@@ -746,8 +871,13 @@ __global__ void __launch_bounds__(THREADS, 1)
                     }
                 }
             }
+            // release the accumulator: one arrival per warp on the MMA issuer's barrier
             fence_before();
-            mbar_arrive(tempty_bar(acc));
+            __syncwarp();
+            if (lane == 0) {
+                if constexpr (PAIR) mbar_arrive_remote(map_to_rank(tempty_bar(acc), 0));
+                else mbar_arrive(tempty_bar(acc));
+            }
             if (++acc == 2) {
                 acc = 0;
                 acc_phase ^= 1u;
@@ -765,11 +895,17 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
     fence_before();
     __syncthreads();
+    if constexpr (PAIR) cluster_sync_all();  // neither CTA leaves while the pair's MMAs run
     fence_after();
     if (warp == 1) {
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base),
-                     "r"(TMEM_COLS)
-                     : "memory");
+        if constexpr (PAIR)
+            asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem_base),
+                         "r"(TMEM_COLS)
+                         : "memory");
+        else
+            asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base),
+                         "r"(TMEM_COLS)
+                         : "memory");
     }
     if constexpr (EPI == EPI_ROUTE) {
         for (int i = threadIdx.x; i < p.hist_n; i += blockDim.x)
@@ -814,6 +950,7 @@ static bool make_map(CUtensorMap* m, const void* base, int64_t inner, int64_t ou
 }
 
 static uint64_t g_wait_ns = 2000000000ull;
+static int g_pairs = 0;  // CTA-pair tiles for the 256-wide M-variable expert GEMMs (off: slower here)
 
 static int sm_count() {
     static int n = 0;
@@ -826,15 +963,17 @@ static int sm_count() {
     return n;
 }
 
-template <int BN, bool B_MN, bool VAR_K, int EPI>
+template <int BN, bool B_MN, bool VAR_K, int EPI, bool PAIR = false>
 static cudaError_t launch(const CUtensorMap& ma, const CUtensorMap& mb, const CUtensorMap& mo0,
                           const CUtensorMap& mo1, const Params& p, int64_t tiles_ub,
                           cudaStream_t s) {
-    auto kern = grouped_gemm_kernel<BN, B_MN, VAR_K, EPI>;
+    auto kern = grouped_gemm_kernel<BN, B_MN, VAR_K, EPI, PAIR>;
+    constexpr int NPAIR = PAIR ? 2 : 1;
+    constexpr int NST = PAIR ? 6 : STAGES;
     const int extra_max = EPI == EPI_ROUTE ? 64 * 64 * 4 : EPI_WARPS * epi_stage_bytes(EPI);
     const int extra = EPI == EPI_ROUTE ? p.hist_n * 4 : EPI_WARPS * epi_stage_bytes(EPI);
-    const int smem_max = STAGES * (BM * BK * 2 + BN * BK * 2) + 1024 + extra_max;
-    const int smem = STAGES * (BM * BK * 2 + BN * BK * 2) + 1024 + extra;
+    const int smem_max = NST * (BM * BK * 2 + BN / NPAIR * BK * 2) + 1024 + extra_max;
+    const int smem = NST * (BM * BK * 2 + BN / NPAIR * BK * 2) + 1024 + extra;
     static bool attr_set = false;
     if (!attr_set) {
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_max);
@@ -842,14 +981,54 @@ static cudaError_t launch(const CUtensorMap& ma, const CUtensorMap& mb, const CU
         attr_set = true;
     }
     if (tiles_ub <= 0) return cudaSuccess;
-    const int grid = (int)std::min<int64_t>(tiles_ub, sm_count());
-    kern<<<grid, THREADS, smem, s>>>(ma, mb, mo0, mo1, p);
-    return cudaGetLastError();
+    if constexpr (PAIR) {
+        // persistent 2-CTA clusters: no more than can be resident at once (a cluster needs
+        // both SMs of a TPC, so fewer than SMs/2 may fit)
+        static int max_clusters = 0;
+        if (!max_clusters) {
+            cudaLaunchConfig_t q = {};
+            q.gridDim = dim3(2 * (sm_count() / 2));
+            q.blockDim = dim3(THREADS);
+            q.dynamicSmemBytes = smem_max;
+            cudaLaunchAttribute qa[1];
+            qa[0].id = cudaLaunchAttributeClusterDimension;
+            qa[0].val.clusterDim.x = 2;
+            qa[0].val.clusterDim.y = 1;
+            qa[0].val.clusterDim.z = 1;
+            q.attrs = qa;
+            q.numAttrs = 1;
+            int n = 0;
+            if (cudaOccupancyMaxActiveClusters(&n, kern, &q) != cudaSuccess || n <= 0) {
+                (void)cudaGetLastError();
+                n = sm_count() / 2;
+            }
+            max_clusters = n;
+        }
+        const int clusters = (int)std::min<int64_t>(tiles_ub, max_clusters);
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(2 * clusters);
+        cfg.blockDim = dim3(THREADS);
+        cfg.dynamicSmemBytes = smem;
+        cfg.stream = s;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = 2;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        return cudaLaunchKernelEx(&cfg, kern, ma, mb, mo0, mo1, p);
+    } else {
+        const int grid = (int)std::min<int64_t>(tiles_ub, sm_count());
+        kern<<<grid, THREADS, smem, s>>>(ma, mb, mo0, mo1, p);
+        return cudaGetLastError();
+    }
 }
 
 }  // namespace tc
 
 void set_wait_limit_ns(uint64_t ns) { tc::g_wait_ns = ns ? ns : 1; }
+void set_gemm_pairs(int on) { tc::g_pairs = on ? 1 : 0; }
 
 // M-variable grouped GEMM (forward, dA, dX).
 cudaError_t launch_gemm_m(const GemmMArgs& g, bool bf16, cudaStream_t s) {
@@ -874,6 +1053,10 @@ cudaError_t launch_gemm_m(const GemmMArgs& g, bool bf16, cudaStream_t s) {
                                           : std::max<int64_t>(g.rows.rows, (int64_t)(g.G - 1) * g.rows.a_stride + g.rows.rows);
     const int64_t mt_ub = g.rows.offsets ? ((int64_t)g.rows.rows + BM - 1) / BM + g.G
                                          : (int64_t)g.G * ((g.rows.rows + BM - 1) / BM);
+    // pair tiles (256 rows)
+    const int64_t pt_ub = g.rows.offsets ? ((int64_t)g.rows.rows + 2 * BM - 1) / (2 * BM) + g.G
+                                         : (int64_t)g.G * ((g.rows.rows + 2 * BM - 1) / (2 * BM));
+    const bool pair = g_pairs != 0;
     // output rows in the 2D view of the outputs
     const int64_t o_rows = g.rows.offsets ? (int64_t)g.rows.rows
                                           : std::max<int64_t>(g.rows.rows, (int64_t)(g.G - 1) * g.rows.out_stride + g.rows.rows);
@@ -886,12 +1069,17 @@ cudaError_t launch_gemm_m(const GemmMArgs& g, bool bf16, cudaStream_t s) {
         if (!make_map(&mb, g.b, g.K, (int64_t)g.G * 2 * F, 128)) return cudaErrorInvalidValue;
         if (!make_map(&mo0, g.out0, 2 * (int64_t)F, o_rows, 0, true)) return cudaErrorInvalidValue;
         if (!make_map(&mo1, g.out1, F, o_rows, 0, true)) return cudaErrorInvalidValue;
+        if (pair) return launch<256, false, false, EPI_SWIGLU_FWD, true>(ma, mb, mo0, mo1, p, pt_ub * (F / 128), s);
         return launch<256, false, false, EPI_SWIGLU_FWD>(ma, mb, mo0, mo1, p, mt_ub * (F / 128), s);
     }
     if (g.epi == EPI_STORE && g.b_kmajor) {  // Y = A W2^T: B = W2[e] as [N=d, K=F]
         p.b_group_rows = g.N;
         if (!make_map(&mo0, g.out0, g.N, o_rows, 0, true)) return cudaErrorInvalidValue;
         if (g.N % 256 == 0) {
+            if (pair) {
+                if (!make_map(&mb, g.b, g.K, (int64_t)g.G * g.N, 128)) return cudaErrorInvalidValue;
+                return launch<256, false, false, EPI_STORE, true>(ma, mb, mo0, mo0, p, pt_ub * (g.N / 256), s);
+            }
             if (!make_map(&mb, g.b, g.K, (int64_t)g.G * g.N, 256)) return cudaErrorInvalidValue;
             return launch<256, false, false, EPI_STORE>(ma, mb, mo0, mo0, p, mt_ub * (g.N / 256), s);
         }
@@ -905,11 +1093,17 @@ cudaError_t launch_gemm_m(const GemmMArgs& g, bool bf16, cudaStream_t s) {
         p.F = g.N;
         if (!make_map(&mo0, g.out0, 2 * (int64_t)g.N, o_rows, 0, true)) return cudaErrorInvalidValue;
         if (!make_map(&mo1, g.aux, 2 * (int64_t)g.N, o_rows, 0, true)) return cudaErrorInvalidValue;
-        if (g.N % 256 == 0) return launch<256, true, false, EPI_SWIGLU_BWD>(ma, mb, mo0, mo1, p, mt_ub * (g.N / 256), s);
+        if (g.N % 256 == 0) {
+            if (pair) return launch<256, true, false, EPI_SWIGLU_BWD, true>(ma, mb, mo0, mo1, p, pt_ub * (g.N / 256), s);
+            return launch<256, true, false, EPI_SWIGLU_BWD>(ma, mb, mo0, mo1, p, mt_ub * (g.N / 256), s);
+        }
         return launch<128, true, false, EPI_SWIGLU_BWD>(ma, mb, mo0, mo1, p, mt_ub * (g.N / 128), s);
     }
     if (!make_map(&mo0, g.out0, g.N, o_rows, 0, true)) return cudaErrorInvalidValue;
-    if (g.N % 256 == 0) return launch<256, true, false, EPI_STORE>(ma, mb, mo0, mo0, p, mt_ub * (g.N / 256), s);
+    if (g.N % 256 == 0) {
+        if (pair) return launch<256, true, false, EPI_STORE, true>(ma, mb, mo0, mo0, p, pt_ub * (g.N / 256), s);
+        return launch<256, true, false, EPI_STORE>(ma, mb, mo0, mo0, p, mt_ub * (g.N / 256), s);
+    }
     return launch<128, true, false, EPI_STORE>(ma, mb, mo0, mo0, p, mt_ub * (g.N / 128), s);
 }
 

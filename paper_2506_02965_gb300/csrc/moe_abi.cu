@@ -142,6 +142,11 @@ moe_status moe_set_wait_limit_ns(uint64_t ns) {
     return MOE_OK;
 }
 
+moe_status moe_set_gemm_pairs(int on) {
+    set_gemm_pairs(on);
+    return MOE_OK;
+}
+
 moe_status moe_workspace_size(const moe_config* cfg, size_t* bytes) {
     moe_status st = check_cfg(cfg);
     if (st) return st;
