@@ -44,11 +44,18 @@ __global__ void __launch_bounds__(DCH) slot_kernel(const int32_t* __restrict__ i
     __shared__ int s_tot[64];
     __shared__ int s_base[64];
     __shared__ unsigned s_bits[64][DCH / 32];
+    constexpr int TAB = 8192;  // chunk-count table staged in shared memory when it fits
+    __shared__ int s_tab[TAB];
     const int c = blockIdx.x;
+    const int64_t ntab = (int64_t)nchunks * E;
+    if (ntab <= TAB) {
+        for (int i = threadIdx.x; i < ntab; i += blockDim.x) s_tab[i] = chunk_counts[i];
+        __syncthreads();
+    }
     for (int e = threadIdx.x; e < E; e += blockDim.x) {
         int pre = 0, tot = 0;
         for (int cc = 0; cc < nchunks; ++cc) {
-            const int v = chunk_counts[(int64_t)cc * E + e];
+            const int v = ntab <= TAB ? s_tab[cc * E + e] : chunk_counts[(int64_t)cc * E + e];
             if (cc < c) pre += v;
             tot += v;
         }

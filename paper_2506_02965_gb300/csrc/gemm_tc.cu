@@ -295,6 +295,17 @@ __host__ __device__ constexpr uint32_t instr_desc() {
            ((B_MN ? 1u : 0u) << 16) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
 }
 
+// Pipeline depth: as many operand stages as fit beside the epilogue's shared memory
+// (staging boxes, or the router's histogram), at most 12.
+__host__ __device__ constexpr int epi_extra_bytes(int epi) {
+    return epi == 3 /* EPI_ROUTE */ ? 64 * 64 * 4 : 4 * (epi == 2 ? 4 : 3) * 2048;
+}
+__host__ __device__ constexpr int num_stages(uint32_t stage_bytes, int epi) {
+    const int budget = 227 * 1024 - 1024 - 1024 - epi_extra_bytes(epi);  // dyn. smem, align, static
+    const int n = budget / (int)stage_bytes;
+    return n > 12 ? 12 : n;
+}
+
 // ------------------------------------------------------------------------ tile geometry
 struct Tile {
     int g;
@@ -397,10 +408,10 @@ __global__ void __launch_bounds__(THREADS, 1)
     constexpr int NPAIR = PAIR ? 2 : 1;
     constexpr int BNL = BN / NPAIR;  // B rows held by this CTA
     constexpr int BMP = BM * NPAIR;  // rows of one (pair) tile
-    constexpr int NST = PAIR ? 6 : STAGES;
     constexpr uint32_t A_BYTES = BM * BK * 2;
     constexpr uint32_t B_BYTES = BNL * BK * 2;
     constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
+    constexpr int NST = num_stages(STAGE_BYTES, EPI);
     constexpr uint32_t IDESC = instr_desc<BN, A_MN, B_MN, BMP>();
     constexpr int TMEM_COLS = (2 * BN <= 32) ? 32 : (2 * BN <= 64) ? 64 : (2 * BN <= 128) ? 128 : (2 * BN <= 256) ? 256 : 512;
 
@@ -969,7 +980,7 @@ static cudaError_t launch(const CUtensorMap& ma, const CUtensorMap& mb, const CU
                           cudaStream_t s) {
     auto kern = grouped_gemm_kernel<BN, B_MN, VAR_K, EPI, PAIR>;
     constexpr int NPAIR = PAIR ? 2 : 1;
-    constexpr int NST = PAIR ? 6 : STAGES;
+    constexpr int NST = num_stages((uint32_t)(BM * BK * 2 + BN / NPAIR * BK * 2), EPI);
     const int extra_max = EPI == EPI_ROUTE ? 64 * 64 * 4 : EPI_WARPS * epi_stage_bytes(EPI);
     const int extra = EPI == EPI_ROUTE ? p.hist_n * 4 : EPI_WARPS * epi_stage_bytes(EPI);
     const int smem_max = NST * (BM * BK * 2 + BN / NPAIR * BK * 2) + 1024 + extra_max;

@@ -66,7 +66,7 @@ class MoELayer:
         self.dw_router = z(P, E, d)
         self.dbias = z(P, E, dtype=f32)
         self.dx = z(T, d)
-        # the router backward runs beside the expert backward on this stream
+        # the aux loss and the router backward run beside the expert GEMMs on this stream
         self.side = torch.cuda.Stream(device=device)
         self.ws_bytes = L.moe_workspace_size(self.cfg)
         self.workspace = torch.empty(max(self.ws_bytes, 16), dtype=torch.uint8, device=device)
@@ -99,19 +99,27 @@ class MoELayer:
     def forward(self, stream=None, mark=None):
         c = self.cfg
         mark = mark or (lambda name: None)
+        main = stream if stream is not None else torch.cuda.current_stream()
         L.moe_route(c, self.x, self.w_router, self.router_bias, self._po(), self.logits,
-                    self.probs, self.topk_idx, self.topk_w, self.counts, stream=stream)
+                    self.probs, self.topk_idx, self.topk_w, self.counts, stream=main)
+        # the aux loss needs only probs and counts: compute it beside the experts
+        fork = torch.cuda.Event()
+        fork.record(main)
+        self.side.wait_event(fork)
         L.moe_aux_loss(c, self.probs, self.counts, self._po(), self.aux_loss, self.aux_coef,
-                       stream=stream)
+                       stream=self.side)
+        aux_done = torch.cuda.Event()
+        aux_done.record(self.side)
         L.moe_dispatch(c, self.topk_idx, self.x, self.offsets, self.slot_of, self.token_of,
-                       self.x_perm, self.workspace, self.ws_bytes, stream=stream)
+                       self.x_perm, self.workspace, self.ws_bytes, stream=main)
         mark("ffn_fwd_begin")
         L.moe_expert_ffn_fwd(c, self.x_perm, self.offsets, self.w1, self.w2, self.h_gu, self.act,
                              self.y_perm, self.x, self.ws1, self.ws2, self.h_gu_sh, self.act_sh,
-                             self.y_sh, stream=stream)
+                             self.y_sh, stream=main)
         mark("ffn_fwd_end")
         L.moe_combine_fwd(c, self.y_perm, self.topk_w, self.slot_of, self.y_sh, self.out,
-                          stream=stream)
+                          stream=main)
+        main.wait_event(aux_done)
 
     def backward(self, stream=None, with_aux: bool = True, mark=None):
         c = self.cfg
