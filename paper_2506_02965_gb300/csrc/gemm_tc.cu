@@ -76,14 +76,16 @@ __device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
 __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
 }
+// One poll: the thread sleeps until the phase completes or at most ~20 us have passed.
+constexpr uint32_t kSuspendHintNs = 20000;
 __device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
     uint32_t ok;
     asm volatile(
         "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
         "selp.u32 %0, 1, 0, p;\n\t}"
         : "=r"(ok)
-        : "r"(bar), "r"(parity)
+        : "r"(bar), "r"(parity), "r"(kSuspendHintNs)
         : "memory");
     return ok != 0;
 }
@@ -93,15 +95,13 @@ __device__ __noinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile i
                                        uint64_t limit_ns) {
     if (mbar_try(bar, parity)) return true;
     const uint64_t t0 = gtimer();
-    for (uint32_t it = 1;; ++it) {
+    for (;;) {
         if (mbar_try(bar, parity)) return true;
-        if ((it & 31u) == 0) {
-            if (*abort_flag) return false;
-            if (gtimer() - t0 > limit_ns) {
-                *abort_flag = 1;
-                record_status(MOE_ERR_TIMEOUT);
-                return false;
-            }
+        if (*abort_flag) return false;
+        if (gtimer() - t0 > limit_ns) {
+            *abort_flag = 1;
+            record_status(MOE_ERR_TIMEOUT);
+            return false;
         }
     }
 }
@@ -131,10 +131,10 @@ __device__ __forceinline__ bool mbar_try_cluster(uint32_t bar, uint32_t parity) 
     uint32_t ok;
     asm volatile(
         "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+        "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2, %3;\n\t"
         "selp.u32 %0, 1, 0, p;\n\t}"
         : "=r"(ok)
-        : "r"(bar), "r"(parity)
+        : "r"(bar), "r"(parity), "r"(kSuspendHintNs)
         : "memory");
     return ok != 0;
 }
@@ -506,15 +506,13 @@ __global__ void __launch_bounds__(THREADS, 1)
         if constexpr (PAIR) {
             if (mbar_try_cluster(bar, parity)) return true;
             const uint64_t t0 = gtimer();
-            for (uint32_t it = 1;; ++it) {
+            for (;;) {
                 if (mbar_try_cluster(bar, parity)) return true;
-                if ((it & 31u) == 0) {
-                    if (*abort_flag) return false;
-                    if (gtimer() - t0 > p.wait_ns) {
-                        *abort_flag = 1;
-                        record_status(MOE_ERR_TIMEOUT);
-                        return false;
-                    }
+                if (*abort_flag) return false;
+                if (gtimer() - t0 > p.wait_ns) {
+                    *abort_flag = 1;
+                    record_status(MOE_ERR_TIMEOUT);
+                    return false;
                 }
             }
         } else {
@@ -556,6 +554,9 @@ __global__ void __launch_bounds__(THREADS, 1)
     fence_after();
     const uint32_t tmem_base = s_tmem;
     const uint64_t limit = p.wait_ns;
+    // drains after an abort wait for work that is already in flight (it completes in
+    // microseconds); their bound does not shrink with a short user wait limit
+    const uint64_t drain_limit = limit > 200000000ull ? limit : 200000000ull;
 
     if (warp == 0) {
         // ------------------------------------------------------------ TMA producer
@@ -622,7 +623,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                     if (issued_phase[s] < 0) continue;
                     const uint64_t t0 = gtimer();
                     while (!mbar_try(full_bar(s), (uint32_t)issued_phase[s]) &&
-                           gtimer() - t0 < limit) {
+                           gtimer() - t0 < drain_limit) {
                     }
                 }
             }
@@ -715,7 +716,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             if constexpr (PAIR) mma_commit_pair(drain_bar, 1);
             else mma_commit(drain_bar);
             const uint64_t t0 = gtimer();
-            while (!mbar_try(drain_bar, 0) && gtimer() - t0 < limit) {
+            while (!mbar_try(drain_bar, 0) && gtimer() - t0 < drain_limit) {
             }
         }
         __syncwarp();
@@ -899,7 +900,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             // loads issued but not consumed (only after an abort): let them land
             for (uint32_t c = gu_chunk; c < gu_issued; ++c) {
                 const uint64_t t0 = gtimer();
-                while (!mbar_try(gu_bar0 + 8u * (c & 1), (c >> 1) & 1) && gtimer() - t0 < limit) {
+                while (!mbar_try(gu_bar0 + 8u * (c & 1), (c >> 1) & 1) && gtimer() - t0 < drain_limit) {
                 }
             }
         }
