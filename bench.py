@@ -69,7 +69,7 @@ def workload_desc(sh):
 
 # --------------------------------------------------------------------------- memory bytes
 def mem_bytes_per_step(sh) -> float:
-    """Algorithmic HBM bytes of the memory-bound stages per step (see DESIGN.md):
+    """Algorithmic HBM bytes of the memory-bound stages per step:
     route read x + write logits/probs/picks; dispatch read x + write x_perm + tables;
     combine read y_perm, w + write out; combine bwd read dout, y_perm + write dy, dw;
     route bwd read probs, dw, x + write dlogits; unpermute read dx_perm (+ dlogits)
@@ -340,7 +340,7 @@ def main():
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": K,
         "warmup": a.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": sh.dtype,
-        "data": "synthetic (seeded numpy PCG64, BASELINE shapes, random-init weights)",
+        "data": "synthetic (seeded numpy PCG64, workload shapes, random-init weights)",
         "config": {"workload": workload_desc(sh), "global_batch": world * sh.T,
                    "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
                    "l2": "flushed (256 MiB write) before every timed step"},

@@ -16,7 +16,7 @@ What it computes (PC-MoE, arXiv 2506.02965):
   * Section 3.2 ("Backward propagation"): the expert host gets the gradient w.r.t.
     the expert output and returns one activation-sized gradient w.r.t. its input.
 
-Readings where the paper is silent (each is listed in the design doc):
+Readings where the paper is silent:
   R1 expert = SwiGLU, E(h) = W2 (silu(W1g h) * (W1u h)), W1 = [W1g; W1u] of shape
      [2F, d] (gate rows first), no biases, no capacity limit;
   R2 optional router bias b (absent unless given);
