@@ -14,6 +14,7 @@ constexpr int DCH = 128;  // tokens per dispatch chunk (one thread each)
 __global__ void __launch_bounds__(DCH) chunk_count_kernel(const int32_t* __restrict__ idx,
                                                           int64_t T, int E, int k,
                                                           int32_t* chunk_counts) {
+    pdl_begin();
     __shared__ int s_cnt[64];
     for (int i = threadIdx.x; i < E; i += blockDim.x) s_cnt[i] = 0;
     __syncthreads();
@@ -40,6 +41,7 @@ __global__ void __launch_bounds__(DCH) slot_kernel(const int32_t* __restrict__ i
                                                    int64_t T, int E, int k, int nchunks,
                                                    int32_t* offsets, int32_t* slot_of,
                                                    int32_t* token_of) {
+    pdl_begin();
     __shared__ int s_pre[64];
     __shared__ int s_tot[64];
     __shared__ int s_base[64];
@@ -106,6 +108,7 @@ template <typename T>
 __global__ void __launch_bounds__(256) gather_kernel(const T* __restrict__ x,
                                                      const int32_t* __restrict__ token_of,
                                                      int64_t TK, int64_t Tn, int d, T* x_perm) {
+    pdl_begin();
     const int lane = threadIdx.x & 31;
     const int64_t r = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
     if (r >= TK) return;
@@ -130,6 +133,7 @@ __global__ void __launch_bounds__(256, 3) combine_fwd_kernel(const T* __restrict
                                                           const int32_t* __restrict__ slot_of,
                                                           const T* __restrict__ y_sh, int S,
                                                           int64_t Tn, int d, int k, T* out) {
+    pdl_begin();
     const int lane = threadIdx.x & 31;
     const int64_t t = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
     if (t >= Tn) return;
@@ -192,6 +196,7 @@ __global__ void __launch_bounds__(256, 3) combine_bwd_kernel(const T* __restrict
                                                           const int32_t* __restrict__ slot_of,
                                                           int64_t Tn, int d, int k, T* dy_perm,
                                                           float* dw) {
+    pdl_begin();
     const int lane = threadIdx.x & 31;
     const int64_t t = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
     if (t >= Tn) return;
@@ -253,16 +258,20 @@ __global__ void __launch_bounds__(256, 3) combine_bwd_kernel(const T* __restrict
 }
 
 // dx[t] = sum_j dx_perm[slot(t,j)] + sum_e dlogits[t,e] W_r[p(t)][e] + sum_s dx_sh[s,t].
-// A block takes UR_TOK tokens of one party and a slab of 64 * VN columns: the party's
-// router rows for the slab and the tokens' dlogits are staged in shared memory; each
-// thread owns VN columns of UR_TOK / 4 tokens.
+// A block takes UR_TOK tokens of one party and a slab of 64 * VN columns; each thread
+// owns VN columns of UR_TOK / 4 tokens. The slot lookups and permuted rows of the first
+// two picks are requested first; while they are in flight the party's router rows for
+// the slab and the tokens' dlogits are staged in shared memory and the router term is
+// accumulated.
 constexpr int UR_TOK = 16;
+constexpr int UR_PRE = 2;  // picks whose rows are loaded before the router term
 
 template <typename T>
 __global__ void __launch_bounds__(256) unpermute_reduce_kernel(
     const T* __restrict__ dx_perm, const int32_t* __restrict__ slot_of,
     const float* __restrict__ dz, const T* __restrict__ wr, const int32_t* __restrict__ po, int P,
     const T* __restrict__ dx_sh, int S, int64_t Tn, int d, int E, int k, T* dx) {
+    pdl_begin();
     constexpr int VN = Vec<T>::N;
     constexpr int SLAB = 64 * VN;
     constexpr int TPT = UR_TOK / 4;  // tokens per thread
@@ -282,6 +291,39 @@ __global__ void __launch_bounds__(256) unpermute_reduce_kernel(
     const int n = (int)min64(UR_TOK, tend - t0);
     const int64_t c0 = (int64_t)blockIdx.y * SLAB;
     const int ncols = (int)min64(SLAB, d - c0);
+    const int cv = threadIdx.x & 63;  // column vector inside the slab
+    const int tg = threadIdx.x >> 6;  // token group
+    const bool active = cv * VN < ncols;
+    const int64_t col = c0 + cv * VN;
+    // slot of pick j of this thread's tokens (-1: no token, or a bad slot, recorded)
+    auto slots_of = [&](int j, int32_t* slot) {
+#pragma unroll
+        for (int i = 0; i < TPT; ++i) {
+            const int tt = tg * TPT + i;
+            slot[i] = (active && tt < n) ? slot_of[(t0 + tt) * k + j] : -1;
+            if (active && tt < n && (slot[i] < 0 || (int64_t)slot[i] >= Tn * k)) {
+                if (cv == 0) record_status(MOE_ERR_DEVICE_CHECK);
+                slot[i] = -1;
+            }
+        }
+    };
+    int32_t pslot[UR_PRE][TPT];
+    uint4 praw[UR_PRE][TPT];
+#pragma unroll
+    for (int j = 0; j < UR_PRE; ++j) {
+        if (j < k) {
+            slots_of(j, pslot[j]);
+        } else {
+#pragma unroll
+            for (int i = 0; i < TPT; ++i) pslot[j][i] = -1;
+        }
+    }
+#pragma unroll
+    for (int j = 0; j < UR_PRE; ++j)
+#pragma unroll
+        for (int i = 0; i < TPT; ++i)
+            if (pslot[j][i] >= 0) praw[j][i] = Vec<T>::raw_load(dx_perm + (int64_t)pslot[j][i] * d + col);
+    // router term: stage dlogits and the party's router rows for this slab
     const T* W = wr + (int64_t)party * E * d;
     for (int i = threadIdx.x; i < UR_TOK * E; i += blockDim.x) {
         const int tt = i / E, e = i % E;
@@ -292,9 +334,7 @@ __global__ void __launch_bounds__(256) unpermute_reduce_kernel(
         if (v * VN < ncols) Vec<T>::raw_store(s_w + e * SLAB + v * VN, Vec<T>::raw_load(W + (int64_t)e * d + c0 + v * VN));
     }
     __syncthreads();
-    const int cv = threadIdx.x & 63;       // column vector inside the slab
-    const int tg = threadIdx.x >> 6;        // token group
-    if (cv * VN >= ncols) return;
+    if (!active) return;
     float acc[TPT][VN];
 #pragma unroll
     for (int i = 0; i < TPT; ++i)
@@ -310,24 +350,7 @@ __global__ void __launch_bounds__(256) unpermute_reduce_kernel(
             for (int q = 0; q < VN; ++q) acc[i][q] = fmaf(zz, wv[q], acc[i][q]);
         }
     }
-    const int64_t col = c0 + cv * VN;
-    // pick by pick: the slot lookups of this thread's tokens, then their rows, in flight
-    // together
-    for (int j = 0; j < k; ++j) {
-        int32_t slot[TPT];
-#pragma unroll
-        for (int i = 0; i < TPT; ++i) {
-            const int tt = tg * TPT + i;
-            slot[i] = tt < n ? slot_of[(t0 + tt) * k + j] : -1;
-            if (tt < n && (slot[i] < 0 || (int64_t)slot[i] >= Tn * k)) {
-                if (cv == 0) record_status(MOE_ERR_DEVICE_CHECK);
-                slot[i] = -1;
-            }
-        }
-        uint4 raw[TPT];
-#pragma unroll
-        for (int i = 0; i < TPT; ++i)
-            if (slot[i] >= 0) raw[i] = Vec<T>::raw_load(dx_perm + (int64_t)slot[i] * d + col);
+    auto add_rows = [&](const int32_t* slot, const uint4* raw) {
 #pragma unroll
         for (int i = 0; i < TPT; ++i) {
             if (slot[i] >= 0) {
@@ -337,6 +360,18 @@ __global__ void __launch_bounds__(256) unpermute_reduce_kernel(
                 for (int q = 0; q < VN; ++q) acc[i][q] += g[q];
             }
         }
+    };
+#pragma unroll
+    for (int j = 0; j < UR_PRE; ++j) add_rows(pslot[j], praw[j]);
+    // remaining picks, one at a time: the slot lookups, then the rows, in flight together
+    for (int j = UR_PRE; j < k; ++j) {
+        int32_t slot[TPT];
+        slots_of(j, slot);
+        uint4 raw[TPT];
+#pragma unroll
+        for (int i = 0; i < TPT; ++i)
+            if (slot[i] >= 0) raw[i] = Vec<T>::raw_load(dx_perm + (int64_t)slot[i] * d + col);
+        add_rows(slot, raw);
     }
 #pragma unroll
     for (int i = 0; i < TPT; ++i) {
@@ -367,19 +402,19 @@ cudaError_t launch_dispatch(const int32_t* topk_idx, const void* x, int64_t T, i
     if (T == 0) {
         return cudaMemsetAsync(offsets, 0, sizeof(int32_t) * (E + 1), s);
     }
-    chunk_count_kernel<<<nch, DCH, 0, s>>>(topk_idx, T, E, k, cc);
+    (void)launch_pdl(chunk_count_kernel, dim3(nch), dim3(DCH), 0, s, topk_idx, T, E, k, cc);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    slot_kernel<<<nch, DCH, 0, s>>>(topk_idx, cc, T, E, k, nch, offsets, slot_of, token_of);
+    (void)launch_pdl(slot_kernel, dim3(nch), dim3(DCH), 0, s, topk_idx, cc, T, E, k, nch, offsets, slot_of, token_of);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     const int64_t TK = T * k;
     const unsigned blocks = (unsigned)((TK + 7) / 8);
     if (bf16)
-        gather_kernel<__nv_bfloat16><<<blocks, 256, 0, s>>>((const __nv_bfloat16*)x, token_of, TK, T,
+        (void)launch_pdl(gather_kernel<__nv_bfloat16>, dim3(blocks), dim3(256), 0, s, (const __nv_bfloat16*)x, token_of, TK, T,
                                                             d, (__nv_bfloat16*)x_perm);
     else
-        gather_kernel<float><<<blocks, 256, 0, s>>>((const float*)x, token_of, TK, T, d,
+        (void)launch_pdl(gather_kernel<float>, dim3(blocks), dim3(256), 0, s, (const float*)x, token_of, TK, T, d,
                                                     (float*)x_perm);
     return cudaGetLastError();
 }
@@ -390,7 +425,7 @@ cudaError_t launch_combine_fwd(const void* y_perm, const float* topk_w, const in
     if (T == 0) return cudaSuccess;
     const unsigned blocks = (unsigned)((T + 7) / 8);
 #define MOE_CF(TT, KM)                                                                           \
-    combine_fwd_kernel<TT, KM><<<blocks, 256, 0, s>>>((const TT*)y_perm, topk_w, slot_of,         \
+    (void)launch_pdl(combine_fwd_kernel<TT, KM>, dim3(blocks), dim3(256), 0, s, (const TT*)y_perm, topk_w, slot_of,         \
                                                       (const TT*)y_sh, S, T, d, k, (TT*)out)
     if (bf16) {
         if (k <= 2) MOE_CF(__nv_bfloat16, 2);
@@ -411,7 +446,7 @@ cudaError_t launch_combine_bwd(const void* dout, const void* y_perm, const float
     if (T == 0) return cudaSuccess;
     const unsigned blocks = (unsigned)((T + 7) / 8);
 #define MOE_CB(TT, KM)                                                                           \
-    combine_bwd_kernel<TT, KM><<<blocks, 256, 0, s>>>((const TT*)dout, (const TT*)y_perm, topk_w, \
+    (void)launch_pdl(combine_bwd_kernel<TT, KM>, dim3(blocks), dim3(256), 0, s, (const TT*)dout, (const TT*)y_perm, topk_w, \
                                                       slot_of, T, d, k, (TT*)dy_perm, dtopk_w)
     if (bf16) {
         if (k <= 2) MOE_CB(__nv_bfloat16, 2);
@@ -445,7 +480,7 @@ cudaError_t launch_unpermute_reduce(const void* dx_perm, const int32_t* slot_of,
             if (e != cudaSuccess) return e;
             attr = true;
         }
-        unpermute_reduce_kernel<__nv_bfloat16><<<grid, 256, smem, s>>>(
+        (void)launch_pdl(unpermute_reduce_kernel<__nv_bfloat16>, dim3(grid), dim3(256), smem, s, 
             (const __nv_bfloat16*)dx_perm, slot_of, dlogits, (const __nv_bfloat16*)w_router, po, P,
             (const __nv_bfloat16*)dx_sh, S, T, d, E, k, (__nv_bfloat16*)dx);
     } else {
@@ -457,7 +492,7 @@ cudaError_t launch_unpermute_reduce(const void* dx_perm, const int32_t* slot_of,
             if (e != cudaSuccess) return e;
             attr = true;
         }
-        unpermute_reduce_kernel<float><<<grid, 256, smem, s>>>(
+        (void)launch_pdl(unpermute_reduce_kernel<float>, dim3(grid), dim3(256), smem, s, 
             (const float*)dx_perm, slot_of, dlogits, (const float*)w_router, po, P,
             (const float*)dx_sh, S, T, d, E, k, (float*)dx);
     }
@@ -497,19 +532,19 @@ cudaError_t launch_dispatch_noalloc(const int32_t* topk_idx, const void* x, int6
     const int nch = (int)((T + DCH - 1) / DCH);
     if ((int64_t)nch * E > kNoAllocScratchInts) return cudaErrorInvalidValue;
     if (T == 0) return cudaMemsetAsync(offsets, 0, sizeof(int32_t) * (E + 1), s);
-    chunk_count_kernel<<<nch, DCH, 0, s>>>(topk_idx, T, E, k, cc);
+    (void)launch_pdl(chunk_count_kernel, dim3(nch), dim3(DCH), 0, s, topk_idx, T, E, k, cc);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    slot_kernel<<<nch, DCH, 0, s>>>(topk_idx, cc, T, E, k, nch, offsets, slot_of, token_of);
+    (void)launch_pdl(slot_kernel, dim3(nch), dim3(DCH), 0, s, topk_idx, cc, T, E, k, nch, offsets, slot_of, token_of);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     const int64_t TK = T * k;
     const unsigned blocks = (unsigned)((TK + 7) / 8);
     if (bf16)
-        gather_kernel<__nv_bfloat16><<<blocks, 256, 0, s>>>((const __nv_bfloat16*)x, token_of, TK, T,
+        (void)launch_pdl(gather_kernel<__nv_bfloat16>, dim3(blocks), dim3(256), 0, s, (const __nv_bfloat16*)x, token_of, TK, T,
                                                             d, (__nv_bfloat16*)x_perm);
     else
-        gather_kernel<float><<<blocks, 256, 0, s>>>((const float*)x, token_of, TK, T, d,
+        (void)launch_pdl(gather_kernel<float>, dim3(blocks), dim3(256), 0, s, (const float*)x, token_of, TK, T, d,
                                                     (float*)x_perm);
     return cudaGetLastError();
 }

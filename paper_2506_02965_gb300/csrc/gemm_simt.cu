@@ -53,6 +53,7 @@ __device__ __forceinline__ int tile_col_to_n(int epi, int c, int n0, int F) {
 }
 
 __global__ void __launch_bounds__(256) gemm_m_simt_kernel(GemmMArgs p) {
+    pdl_begin();
     __shared__ float As[SB_K][SB_M + 4];
     __shared__ float Bs[SB_K][SB_N + 4];
     int g, m0, mrows;
@@ -143,6 +144,7 @@ __global__ void __launch_bounds__(256) gemm_m_simt_kernel(GemmMArgs p) {
 }
 
 __global__ void __launch_bounds__(256) gemm_k_simt_kernel(GemmKArgs p) {
+    pdl_begin();
     __shared__ float As[SB_K][SB_M + 4];
     __shared__ float Bs[SB_K][SB_N + 4];
     const int g = blockIdx.z;
@@ -214,13 +216,13 @@ cudaError_t launch_gemm_m_simt(const GemmMArgs& g, cudaStream_t s) {
     }
     if (mt_ub <= 0) return cudaSuccess;
     dim3 grid((ncols + per - 1) / per, (unsigned)mt_ub);
-    gemm_m_simt_kernel<<<grid, 256, 0, s>>>(g);
+    (void)launch_pdl(gemm_m_simt_kernel, dim3(grid), dim3(256), 0, s, g);
     return cudaGetLastError();
 }
 
 cudaError_t launch_gemm_k_simt(const GemmKArgs& g, cudaStream_t s) {
     dim3 grid((g.N + SB_N - 1) / SB_N, (g.M + SB_M - 1) / SB_M, g.G);
-    gemm_k_simt_kernel<<<grid, 256, 0, s>>>(g);
+    (void)launch_pdl(gemm_k_simt_kernel, dim3(grid), dim3(256), 0, s, g);
     return cudaGetLastError();
 }
 

@@ -28,12 +28,12 @@ constexpr int EPI_WARPS = 4;
 constexpr int THREADS = 64 + 32 * EPI_WARPS;  // TMA warp, MMA warp, epilogue warps
 constexpr int EPI_BOX = 32;                     // TMA-store box: 32 columns x 32 rows (bf16)
 constexpr int EPI_BUF_BYTES = EPI_BOX * EPI_BOX * 2;
-// per epilogue warp: up to 3 output boxes, or for the SwiGLU backward 2 x (G, U) boxes
-constexpr int EPI_STAGE_BYTES = 3 * EPI_BUF_BYTES;
-constexpr int EPI_STAGE_BYTES_BWD = 4 * EPI_BUF_BYTES;
-__host__ __device__ constexpr int epi_stage_bytes(int epi) {
-    return epi == EPI_SWIGLU_BWD ? EPI_STAGE_BYTES_BWD : EPI_STAGE_BYTES;
-}
+// per epilogue warp: a ring of 4 output boxes (each box leaves by its own TMA store, so
+// up to 3 stores are in flight while the next box is written), or for the SwiGLU
+// backward 2 x (G, U) boxes
+constexpr int EPI_NBUF = 4;
+constexpr int EPI_STAGE_BYTES = EPI_NBUF * EPI_BUF_BYTES;
+__host__ __device__ constexpr int epi_stage_bytes(int) { return EPI_STAGE_BYTES; }
 constexpr int MAX_GROUPS = 128;
 
 struct Params {
@@ -188,6 +188,11 @@ __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.comm
 __device__ __forceinline__ void bulk_wait_read0() {
     asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
 }
+// wait until at most N of this thread's bulk groups are still reading shared memory
+template <int N>
+__device__ __forceinline__ void bulk_wait_read() {
+    asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
+}
 __device__ __forceinline__ void bulk_wait0() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 __device__ __forceinline__ void fence_proxy_async() {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -298,7 +303,7 @@ __host__ __device__ constexpr uint32_t instr_desc() {
 // Pipeline depth: as many operand stages as fit beside the epilogue's shared memory
 // (staging boxes, or the router's histogram), at most 12.
 __host__ __device__ constexpr int epi_extra_bytes(int epi) {
-    return epi == 3 /* EPI_ROUTE */ ? 64 * 64 * 4 : 4 * (epi == 2 ? 4 : 3) * 2048;
+    return epi == 3 /* EPI_ROUTE */ ? 64 * 64 * 4 : 4 * EPI_STAGE_BYTES;
 }
 __host__ __device__ constexpr int num_stages(uint32_t stage_bytes, int epi) {
     const int budget = 227 * 1024 - 1024 - 1024 - epi_extra_bytes(epi);  // dyn. smem, align, static
@@ -404,6 +409,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                         const __grid_constant__ CUtensorMap tmB,
                         const __grid_constant__ CUtensorMap tmO0,
                         const __grid_constant__ CUtensorMap tmO1, const Params p) {
+    pdl_begin();
     constexpr bool A_MN = VAR_K;
     constexpr int NPAIR = PAIR ? 2 : 1;
     constexpr int BNL = BN / NPAIR;  // B rows held by this CTA
@@ -731,6 +737,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         const uint32_t stg_u32 = smem_u32(stg);
         int acc = 0;
         uint32_t acc_phase = 0;
+        uint32_t box_seq = 0;  // output boxes this warp has staged (ring position)
         // SwiGLU backward: TMA loads of G/U chunk boxes into two staging buffers
         const uint32_t gu_bar0 = bar0 + 8u * (2 * NST + 5 + 2 * (warp - 2));
         uint32_t gu_issued = 0;  // chunks whose loads were issued (this warp)
@@ -767,16 +774,20 @@ __global__ void __launch_bounds__(THREADS, 1)
             auto emit = [&](int nout, const float* const* vals, const CUtensorMap* const* maps,
                             const int* cols, __nv_bfloat16* const* direct) {
                 if (full_box) {
-                    if (lane == 0) bulk_wait_read0();  // staging free again
-                    __syncwarp();
-                    for (int o = 0; o < nout; ++o)
-                        store_row32_sw64(stg + o * EPI_BUF_BYTES + lane * 64, lane, vals[o]);
-                    fence_proxy_async();
-                    __syncwarp();
-                    if (lane == 0) {
-                        for (int o = 0; o < nout; ++o)
-                            tma_store_2d(maps[o], stg_u32 + o * EPI_BUF_BYTES, cols[o], (int)grow0);
-                        bulk_commit();
+#pragma unroll
+                    for (int o = 0; o < nout; ++o) {
+                        const uint32_t b = box_seq & (EPI_NBUF - 1);
+                        // the store that last used box b (EPI_NBUF boxes ago) has read it
+                        if (lane == 0) bulk_wait_read<EPI_NBUF - 1>();
+                        __syncwarp();
+                        store_row32_sw64(stg + b * EPI_BUF_BYTES + lane * 64, lane, vals[o]);
+                        fence_proxy_async();
+                        __syncwarp();
+                        if (lane == 0) {
+                            tma_store_2d(maps[o], stg_u32 + b * EPI_BUF_BYTES, cols[o], (int)grow0);
+                            bulk_commit();
+                        }
+                        ++box_seq;
                     }
                 } else if (valid) {
                     for (int o = 0; o < nout; ++o) store_row32(direct[o], vals[o]);
@@ -1022,17 +1033,19 @@ static cudaError_t launch(const CUtensorMap& ma, const CUtensorMap& mb, const CU
         cfg.blockDim = dim3(THREADS);
         cfg.dynamicSmemBytes = smem;
         cfg.stream = s;
-        cudaLaunchAttribute attr[1];
+        cudaLaunchAttribute attr[2];
         attr[0].id = cudaLaunchAttributeClusterDimension;
         attr[0].val.clusterDim.x = 2;
         attr[0].val.clusterDim.y = 1;
         attr[0].val.clusterDim.z = 1;
+        attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[1].val.programmaticStreamSerializationAllowed = 1;
         cfg.attrs = attr;
-        cfg.numAttrs = 1;
+        cfg.numAttrs = 2;
         return cudaLaunchKernelEx(&cfg, kern, ma, mb, mo0, mo1, p);
     } else {
         const int grid = (int)std::min<int64_t>(tiles_ub, sm_count());
-        kern<<<grid, THREADS, smem, s>>>(ma, mb, mo0, mo1, p);
+        (void)launch_pdl(kern, dim3(grid), dim3(THREADS), smem, s, ma, mb, mo0, mo1, p);
         return cudaGetLastError();
     }
 }

@@ -27,6 +27,34 @@ static inline cudaError_t tu_status_read_clear(cudaStream_t s, int* code) {
     return cudaStreamSynchronize(s);
 }
 
+// ---------------------------------------------------------------- dependent launches
+// Every kernel of the layer is launched with programmatic stream serialization (see
+// launch_pdl): it may be scheduled while the kernel before it in the stream is still
+// finishing. pdl_begin() is the first statement of every kernel body. It first allows
+// the next kernel of the stream to be scheduled (once every block of this grid has
+// started), then waits until the previous kernel has completed and its writes are
+// visible, so no global memory is read or written before its producer is done.
+__device__ __forceinline__ void pdl_begin() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
+template <typename... KArgs, typename... Args>
+static inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                                     cudaStream_t s, Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, args...);
+}
+
 // ---------------------------------------------------------------- element access
 template <typename T> struct Elem;
 template <> struct Elem<float> {

@@ -80,6 +80,7 @@ __global__ void __launch_bounds__(256) route_kernel(
     const float* __restrict__ logits_in, const int32_t* __restrict__ po, int P, int64_t Tn,
     int d, int E, int k, int normalize, float* logits, float* probs, int32_t* topk_idx,
     float* topk_w, int32_t* counts) {
+    pdl_begin();
     extern __shared__ int s_hist[];  // [P*E]
     for (int i = threadIdx.x; i < P * E; i += blockDim.x) s_hist[i] = 0;
     __syncthreads();
@@ -181,6 +182,7 @@ __global__ void __cluster_dims__(AUX_CLUSTER, 1, 1) __launch_bounds__(AUX_THREAD
     aux_loss_kernel(const float* __restrict__ probs, const int32_t* __restrict__ counts,
                     const int32_t* __restrict__ po, int64_t Tn, int E, int k, float alpha,
                     float* loss, float* coef) {
+    pdl_begin();
     __shared__ float s_part[AUX_THREADS];
     __shared__ float s_col[64];
     cg::cluster_group cluster = cg::this_cluster();
@@ -254,6 +256,7 @@ __global__ void __launch_bounds__(256) dlogits_kernel(
     const float* __restrict__ topk_w, const float* __restrict__ dtopk_w,
     const float* __restrict__ aux_coef, const int32_t* __restrict__ po, int P, int64_t Tn, int E,
     int k, int normalize, float* dlogits) {
+    pdl_begin();
     const int lane = threadIdx.x & 31;
     const int64_t t = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
     if (t >= Tn) return;
@@ -295,6 +298,7 @@ template <typename T>
 __global__ void __launch_bounds__(2 * RB_HALF) route_bwd_partial_kernel(
     const T* __restrict__ x, const float* __restrict__ dz, const int32_t* __restrict__ po, int P,
     int64_t Tn, int d, int E, float* part_dw, float* part_db) {
+    pdl_begin();
     constexpr int VN = Vec<T>::N;
     constexpr int SLAB = RB_HALF * VN;
     __shared__ float s_dz[RB_CH][RB_ET];
@@ -376,6 +380,7 @@ template <typename T>
 __global__ void __launch_bounds__(RR_OUT * RR_GRP) route_bwd_reduce_kernel(
     const float* __restrict__ part_dw, const float* __restrict__ part_db,
     const int32_t* __restrict__ po, int P, int64_t Tn, int d, int E, T* dw_router, float* dbias) {
+    pdl_begin();
     __shared__ float s_sum[RR_GRP][RR_OUT];
     const int o = threadIdx.x % RR_OUT, g = threadIdx.x / RR_OUT;
     const int64_t i = (int64_t)blockIdx.x * RR_OUT + o;
@@ -438,7 +443,7 @@ static cudaError_t launch_route_t(const RouteArgs& a, cudaStream_t s) {
     const T* x = (const T*)a.x;
     const T* wr = (const T*)a.w_router;
 #define MOE_ROUTE_CASE(EM, TP)                                                                   \
-    route_kernel<T, EM, TP, FROM><<<blocks, 256, smem, s>>>(                                      \
+    (void)launch_pdl(route_kernel<T, EM, TP, FROM>, dim3(blocks), dim3(256), smem, s,                                       \
         x, wr, a.bias, a.logits_in, a.po, a.P, a.T, a.d, E, a.k, a.normalize, a.logits, a.probs, \
         a.topk_idx, a.topk_w, a.counts)
     if constexpr (FROM) {
@@ -467,7 +472,7 @@ cudaError_t launch_route(const RouteArgs& a, bool bf16, bool from_logits, cudaSt
 cudaError_t launch_aux_loss(const float* probs, const int32_t* counts, const int32_t* po, int P,
                             int64_t T, int E, int k, float alpha, float* loss, float* coef,
                             cudaStream_t s) {
-    aux_loss_kernel<<<P * AUX_CLUSTER, AUX_THREADS, 0, s>>>(probs, counts, po, T, E, k, alpha, loss, coef);
+    (void)launch_pdl(aux_loss_kernel, dim3(P * AUX_CLUSTER), dim3(AUX_THREADS), 0, s, probs, counts, po, T, E, k, alpha, loss, coef);
     return cudaGetLastError();
 }
 
@@ -483,7 +488,7 @@ static cudaError_t launch_route_bwd_t(const RouteBwdArgs& a, void* ws, cudaStrea
     float* part_db = part_dw + nch * a.E * a.d;
     if (a.T > 0) {
         const unsigned blocks = (unsigned)((a.T + 7) / 8);
-        dlogits_kernel<<<blocks, 256, 0, s>>>(a.probs, a.topk_idx, a.topk_w, a.dtopk_w, a.aux_coef,
+        (void)launch_pdl(dlogits_kernel, dim3(blocks), dim3(256), 0, s, a.probs, a.topk_idx, a.topk_w, a.dtopk_w, a.aux_coef,
                                               a.po, a.P, a.T, a.E, a.k, a.normalize, a.dlogits);
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
@@ -498,12 +503,12 @@ static cudaError_t launch_route_bwd_t(const RouteBwdArgs& a, void* ws, cudaStrea
         if (e != cudaSuccess) return e;
         attr = true;
     }
-    route_bwd_partial_kernel<T><<<grid, 2 * RB_HALF, smem, s>>>((const T*)a.x, a.dlogits, a.po,
+    (void)launch_pdl(route_bwd_partial_kernel<T>, dim3(grid), dim3(2 * RB_HALF), smem, s, (const T*)a.x, a.dlogits, a.po,
                                                                 a.P, a.T, a.d, a.E, part_dw, part_db);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     const int64_t total = (int64_t)a.P * a.E * a.d;
-    route_bwd_reduce_kernel<T><<<(unsigned)((total + RR_OUT - 1) / RR_OUT), RR_OUT * RR_GRP, 0, s>>>(
+    (void)launch_pdl(route_bwd_reduce_kernel<T>, dim3((unsigned)((total + RR_OUT - 1) / RR_OUT)), dim3(RR_OUT * RR_GRP), 0, s, 
         part_dw, part_db, a.po, a.P, a.T, a.d, a.E, (T*)a.dw_router, a.dbias);
     return cudaGetLastError();
 }
