@@ -238,11 +238,18 @@ moe_status moe_device_status(moe_stream_t stream, int32_t* code /* HOST out */);
 moe_status moe_set_wait_limit_ns(uint64_t ns);
 
 /* Tile shape of the 256-wide expert GEMMs whose rows vary per expert (forward, dA,
- * dX). on = 0 (default): one CTA per 128 x 256 tile; on = 1: a pair of CTAs on two SMs
- * computes each 256 x 256 tile with tcgen05 cta_group::2 MMAs, each SM holding half of
- * the B operand (measured slower than on = 0 on GB300 for these shapes). Results agree
- * up to fp32 summation order. */
-moe_status moe_set_gemm_pairs(int on);
+ * dX), for all later calls of this process. A CTA-pair tile is 256 x 256, computed by
+ * two CTAs on two SMs with tcgen05 cta_group::2 MMAs, each SM holding half of the B
+ * operand (half the operand traffic per SM of a single-CTA 128 x 256 tile), but twice
+ * as few tiles share the SMs, so a launch with few tiles loses to its last round.
+ *   MOE_PAIRS_OFF  (0): single-CTA tiles everywhere;
+ *   MOE_PAIRS_ALL  (1): pair tiles for every such GEMM;
+ *   MOE_PAIRS_AUTO (2, default): pair tiles where a launch has at least four rounds of
+ *                   them and its epilogue is not the SwiGLU backward (which, not the
+ *                   operand feed, bounds the dA GEMM).
+ * Results agree up to fp32 summation order. Any other mode: MOE_ERR_INVALID_ARG. */
+enum { MOE_PAIRS_OFF = 0, MOE_PAIRS_ALL = 1, MOE_PAIRS_AUTO = 2 };
+moe_status moe_set_gemm_pairs(int mode);
 
 const char* moe_status_string(moe_status s);
 /* Reason for the last MOE_ERR_INVALID_ARG / MOE_ERR_CUDA returned on this thread. */

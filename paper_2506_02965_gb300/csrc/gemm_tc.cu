@@ -117,12 +117,6 @@ __device__ __forceinline__ uint32_t map_to_rank(uint32_t addr, uint32_t rank) {
     asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
     return r;
 }
-__device__ __forceinline__ void mbar_expect_tx_remote(uint32_t cluster_bar, uint32_t bytes) {
-    asm volatile("mbarrier.arrive.expect_tx.release.cluster.shared::cluster.b64 _, [%0], %1;" ::"r"(
-                     cluster_bar),
-                 "r"(bytes)
-                 : "memory");
-}
 __device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_bar) {
     asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_bar)
                  : "memory");
@@ -528,7 +522,7 @@ __global__ void __launch_bounds__(THREADS, 1)
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < NST; ++s) {
-            mbar_init(full_bar(s), NPAIR);  // one producer arrival per CTA of the pair
+            mbar_init(full_bar(s), 1);  // the (leader's) producer arms it for both CTAs' bytes
             mbar_init(empty_bar(s), 1);
         }
         for (int a = 0; a < 2; ++a) {
@@ -587,8 +581,16 @@ __global__ void __launch_bounds__(THREADS, 1)
                     const uint32_t sa = ring + stage * STAGE_BYTES;
                     const uint32_t sb = sa + A_BYTES;
                     const uint32_t fb = PAIR ? map_to_rank(full_bar(stage), 0) : full_bar(stage);
-                    if constexpr (PAIR) mbar_expect_tx_remote(fb, STAGE_BYTES);
-                    else mbar_expect_tx(fb, STAGE_BYTES);
+                    // In a pair only the leader arrives, expecting the bytes of both CTAs: the
+                    // peer's copies complete on the leader's barrier without an arrival (a
+                    // cluster-scope arrive per stage cost the producers most of their time). The
+                    // peer reuses a stage only after the leader's MMAs released it, so its bytes
+                    // always count towards the phase the leader arms.
+                    if constexpr (PAIR) {
+                        if (rank == 0) mbar_expect_tx(full_bar(stage), NPAIR * STAGE_BYTES);
+                    } else {
+                        mbar_expect_tx(fb, STAGE_BYTES);
+                    }
                     const int k0 = kb * BK;
                     if (!A_MN) {
                         load(sa, &tmA, fb, k0, (int)(ti.a_row + ti.m0));
@@ -973,7 +975,7 @@ static bool make_map(CUtensorMap* m, const void* base, int64_t inner, int64_t ou
 }
 
 static uint64_t g_wait_ns = 2000000000ull;
-static int g_pairs = 0;  // CTA-pair tiles for the 256-wide M-variable expert GEMMs (off: slower here)
+static int g_pairs = MOE_PAIRS_AUTO;  // CTA-pair tiles for the 256-wide M-variable expert GEMMs
 
 static int sm_count() {
     static int n = 0;
@@ -1053,7 +1055,7 @@ static cudaError_t launch(const CUtensorMap& ma, const CUtensorMap& mb, const CU
 }  // namespace tc
 
 void set_wait_limit_ns(uint64_t ns) { tc::g_wait_ns = ns ? ns : 1; }
-void set_gemm_pairs(int on) { tc::g_pairs = on ? 1 : 0; }
+void set_gemm_pairs(int mode) { tc::g_pairs = mode; }
 
 // M-variable grouped GEMM (forward, dA, dX).
 cudaError_t launch_gemm_m(const GemmMArgs& g, bool bf16, cudaStream_t s) {
@@ -1081,7 +1083,13 @@ cudaError_t launch_gemm_m(const GemmMArgs& g, bool bf16, cudaStream_t s) {
     // pair tiles (256 rows)
     const int64_t pt_ub = g.rows.offsets ? ((int64_t)g.rows.rows + 2 * BM - 1) / (2 * BM) + g.G
                                          : (int64_t)g.G * ((g.rows.rows + 2 * BM - 1) / (2 * BM));
-    const bool pair = g_pairs != 0;
+    // pair tiles where they fill at least four rounds of the SMs (the last, partly empty
+    // round then costs little) and the operand feed, not the epilogue, bounds the tile
+    const int64_t pair_tiles = pt_ub * (g.N / 256);
+    const bool pair = g.N % 256 == 0 &&
+                      (g_pairs == MOE_PAIRS_ALL ||
+                       (g_pairs == MOE_PAIRS_AUTO && g.epi != EPI_SWIGLU_BWD &&
+                        pair_tiles >= 4 * (int64_t)(sm_count() / 2)));
     // output rows in the 2D view of the outputs
     const int64_t o_rows = g.rows.offsets ? (int64_t)g.rows.rows
                                           : std::max<int64_t>(g.rows.rows, (int64_t)(g.G - 1) * g.rows.out_stride + g.rows.rows);

@@ -142,8 +142,10 @@ moe_status moe_set_wait_limit_ns(uint64_t ns) {
     return MOE_OK;
 }
 
-moe_status moe_set_gemm_pairs(int on) {
-    set_gemm_pairs(on);
+moe_status moe_set_gemm_pairs(int mode) {
+    if (mode != MOE_PAIRS_OFF && mode != MOE_PAIRS_ALL && mode != MOE_PAIRS_AUTO)
+        return fail(MOE_ERR_INVALID_ARG, "pair mode must be MOE_PAIRS_OFF, _ALL or _AUTO");
+    set_gemm_pairs(mode);
     return MOE_OK;
 }
 

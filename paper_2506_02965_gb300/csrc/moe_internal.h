@@ -123,7 +123,7 @@ struct GemmKArgs {
 cudaError_t launch_gemm_m(const GemmMArgs& g, bool bf16, cudaStream_t s);
 cudaError_t launch_gemm_k(const GemmKArgs& g, bool bf16, cudaStream_t s);
 void set_wait_limit_ns(uint64_t ns);
-void set_gemm_pairs(int on);
+void set_gemm_pairs(int mode);  // MOE_PAIRS_*
 cudaError_t gemm_status(cudaStream_t s, int* code);
 cudaError_t simt_status(cudaStream_t s, int* code);
 

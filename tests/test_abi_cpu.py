@@ -54,6 +54,14 @@ def test_status_strings_and_version(L):
     assert "sm_103a" in L.moe_version()
 
 
+def test_pair_mode_checked_on_host(L):
+    for mode in (0, 1, 2):
+        L.moe_set_gemm_pairs(mode)
+    with pytest.raises(L.MoEError, match="pair mode"):
+        L.moe_set_gemm_pairs(3)
+    L.moe_set_gemm_pairs(2)  # the default
+
+
 def test_workspace_size_is_host_only(L):
     cfg = L.make_config(4096, 1024, 16, 2816, 2)
     n = L.moe_workspace_size(cfg)

@@ -118,10 +118,11 @@ def test_expert_ffn_is_deterministic(L):
         assert torch.equal(a, b)
 
 
-@pytest.mark.parametrize("pairs", [0, 1])
+@pytest.mark.parametrize("pairs", [0, 1, 2])
 def test_expert_ffn_single_cta_and_pair_tiles(L, pairs):
-    """The 256-wide M-variable GEMMs in both tile shapes: one CTA per 128x256 tile, or a
-    CTA pair per 256x256 tile (ragged experts, an empty expert, a skewed split)."""
+    """The 256-wide M-variable GEMMs in every tile mode: one CTA per 128x256 tile, a CTA
+    pair per 256x256 tile, or the automatic choice per launch (ragged experts, an empty
+    expert, a skewed split)."""
     L.moe_set_gemm_pairs(pairs)
     try:
         for case in [(777, 512, 8, 512, 2, "skewed", "bf16", 0, 0),
@@ -129,4 +130,4 @@ def test_expert_ffn_single_cta_and_pair_tiles(L, pairs):
                      (1024, 1024, 16, 2816, 2, "uniform", "bf16", 0, 0)]:
             test_expert_ffn_fwd_bwd(L, case)
     finally:
-        L.moe_set_gemm_pairs(0)
+        L.moe_set_gemm_pairs(2)
