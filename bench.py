@@ -299,12 +299,7 @@ def main():
         for i in range(Ke):
             flush.fill_(i & 0xFF)
             e0.record(stream)
-            lay.x.copy_(hx, non_blocking=True)
-            lay.dout.copy_(hd, non_blocking=True)
-            lay.step()
-            ho.copy_(lay.out, non_blocking=True)
-            hdx.copy_(lay.dx, non_blocking=True)
-            hloss.copy_(lay.aux_loss, non_blocking=True)
+            lay.step_host(hx, hd, ho, hdx, hloss, stream=stream)
             e1.record(stream)
             e1.synchronize()
             times.append(e0.elapsed_time(e1))

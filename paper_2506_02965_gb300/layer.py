@@ -68,6 +68,8 @@ class MoELayer:
         self.dx = z(T, d)
         # the aux loss and the router backward run beside the expert GEMMs on this stream
         self.side = torch.cuda.Stream(device=device)
+        # host<->device copies that overlap the passes (step_host)
+        self.copy_stream = torch.cuda.Stream(device=device)
         self.ws_bytes = L.moe_workspace_size(self.cfg)
         self.workspace = torch.empty(max(self.ws_bytes, 16), dtype=torch.uint8, device=device)
 
@@ -152,6 +154,39 @@ class MoELayer:
         the boundaries of the expert-GEMM calls: ffn_fwd_begin/end, ffn_bwd_begin/end."""
         self.forward(stream, mark=mark)
         self.backward(stream, mark=mark)
+
+    def step_host(self, hx, hdout, hout, hdx, hloss, stream=None):
+        """One fwd+bwd pass fed from host memory: x and dOut are copied in from the host
+        tensors ``hx``, ``hdout`` (pinned for asynchronous copies), out, dx and the aux loss
+        are copied back into ``hout``, ``hdx``, ``hloss``. Only x has to arrive before the
+        forward and only dx leaves after the backward: dOut's upload runs beside the
+        forward and out's download beside the backward, on a copy stream. All copies are
+        ordered before the stream's later work, so the next call may reuse every buffer.
+        """
+        main = stream if stream is not None else torch.cuda.current_stream()
+        start = torch.cuda.Event()
+        start.record(main)  # the previous pass on this stream is done with dout and out
+        with torch.cuda.stream(main):
+            self.x.copy_(hx, non_blocking=True)
+        self.copy_stream.wait_event(start)
+        with torch.cuda.stream(self.copy_stream):
+            self.dout.copy_(hdout, non_blocking=True)
+        dout_in = torch.cuda.Event()
+        dout_in.record(self.copy_stream)
+        self.forward(main)
+        fwd_done = torch.cuda.Event()
+        fwd_done.record(main)
+        self.copy_stream.wait_event(fwd_done)
+        with torch.cuda.stream(self.copy_stream):
+            hout.copy_(self.out, non_blocking=True)
+        out_back = torch.cuda.Event()
+        out_back.record(self.copy_stream)
+        main.wait_event(dout_in)
+        self.backward(main)
+        with torch.cuda.stream(main):
+            hdx.copy_(self.dx, non_blocking=True)
+            hloss.copy_(self.aux_loss, non_blocking=True)
+        main.wait_event(out_back)
 
     def kernels_per_step(self) -> int:
         """CUDA kernels this library launches per step (memsets not counted):

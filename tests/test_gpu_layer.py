@@ -100,6 +100,36 @@ def test_layer_is_deterministic(L):
         assert torch.equal(getattr(a, n), getattr(b, n)), n
 
 
+def test_step_from_host_buffers_matches_device_step(L):
+    """step_host (x and dOut from pinned host memory, overlapped copies, results back to
+    the host) gives the same bits as a step on device-resident inputs, on three steps in
+    a row with different inputs each step (so a copy racing a pass would show)."""
+    sh = mi.SHAPES[2].with_(T=1024)
+    lay = MoELayer(sh)
+    lay.load(mi.make_inputs(sh))
+    ref = MoELayer(sh)
+    ref.load(mi.make_inputs(sh))
+    hx = torch.empty(sh.T, sh.d_model, dtype=lay.dt).pin_memory()
+    hd, ho, hdx = torch.empty_like(hx).pin_memory(), torch.empty_like(hx).pin_memory(), \
+        torch.empty_like(hx).pin_memory()
+    hloss = torch.empty(sh.n_parties, dtype=torch.float32).pin_memory()
+    for i in range(3):
+        inp = mi.make_inputs(sh.with_(seed=sh.seed + 100 + i), with_weights=False)
+        hx.copy_(torch.from_numpy(inp["x"]).to(lay.dt))
+        hd.copy_(torch.from_numpy(inp["dout"]).to(lay.dt))
+        lay.step_host(hx, hd, ho, hdx, hloss)
+        torch.cuda.synchronize()
+        ref.x.copy_(hx)
+        ref.dout.copy_(hd)
+        ref.step()
+        torch.cuda.synchronize()
+        assert torch.equal(ho, ref.out.cpu()), i
+        assert torch.equal(hdx, ref.dx.cpu()), i
+        assert torch.equal(hloss, ref.aux_loss.cpu()), i
+        assert torch.equal(lay.dw1, ref.dw1), i
+    assert status(L) == 0
+
+
 def test_layer_empty_batch(L):
     sh = mi.MoEShape("empty", 0, 256, 8, 256, 2, "bf16")
     lay = MoELayer(sh)
