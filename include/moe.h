@@ -208,25 +208,30 @@ moe_status moe_expert_ffn_bwd(const moe_config* cfg, const void* x_perm, const i
  *   dlogits[t,e] = probs[t,e] * (dp[t,e] - <dp[t], probs[t]>)   [T,E] f32 out
  *   dw_router[p] = sum_{t in p} dlogits[t]^T x[t]                [P,E,d] dtype out
  *   dbias[p]     = sum_{t in p} dlogits[t]                       [P,E] f32 out or NULL
- * aux_coef may be NULL (no aux term). Deterministic: partial sums go to the
- * workspace and are reduced in a fixed order.
+ *   dx_router[t] = dlogits[t] W_r[p(t)]  (the router's share of the input gradient)
+ *                                                               [T,d] dtype out or NULL
+ * aux_coef may be NULL (no aux term). bf16: the two products run on the tensor cores
+ * with dlogits rounded to bf16 as their operand (fp32 accumulation); fp32: CUDA cores.
+ * Deterministic: partial sums go to the workspace and are reduced in a fixed order.
  */
 moe_status moe_route_bwd(const moe_config* cfg, const void* x, const void* w_router,
                          const float* probs, const int32_t* topk_idx, const float* topk_w,
                          const float* dtopk_w, const float* aux_coef,
                          const int32_t* party_offsets, float* dlogits, void* dw_router,
-                         float* dbias, void* workspace, size_t workspace_bytes,
-                         moe_stream_t stream);
+                         float* dbias, void* dx_router, void* workspace,
+                         size_t workspace_bytes, moe_stream_t stream);
 
 /*
  * Input gradient of the layer: the returned expert-input gradients summed per token
- * (Sec. 3.2), plus the router's share and the shared experts' share:
- *   dx[t] = sum_j dx_perm[slot_of[t*k+j]] + dlogits[t] W_r[p(t)] + sum_s dx_sh[s,t]
- *   dx [T,d] dtype out (overwritten; fp32 accumulation). dx_sh NULL when S == 0.
+ * (Sec. 3.2), plus the router's share (dx_router from moe_route_bwd) and the shared
+ * experts' share:
+ *   dx[t] = sum_j dx_perm[slot_of[t*k+j]] + dx_router[t] + sum_s dx_sh[s,t]
+ *   dx [T,d] dtype out (overwritten; fp32 accumulation). dx_router NULL: no router
+ *   term. dx_sh NULL when S == 0. A slot outside [0, T*k) is skipped and recorded as
+ *   MOE_ERR_DEVICE_CHECK (moe_device_status).
  */
 moe_status moe_dispatch_bwd(const moe_config* cfg, const void* dx_perm, const int32_t* slot_of,
-                            const float* dlogits, const void* w_router,
-                            const int32_t* party_offsets, const void* dx_sh, void* dx,
+                            const void* dx_router, const void* dx_sh, void* dx,
                             moe_stream_t stream);
 
 /* Synchronises `stream`, returns the first error code any kernel recorded since the

@@ -70,8 +70,8 @@ _SIGS = {
     "moe_combine_fwd": [_CFG] + [P] * 6,
     "moe_combine_bwd": [_CFG] + [P] * 7,
     "moe_expert_ffn_bwd": [_CFG] + [P] * 22,
-    "moe_route_bwd": [_CFG] + [P] * 12 + [ctypes.c_size_t, P],
-    "moe_dispatch_bwd": [_CFG] + [P] * 8,
+    "moe_route_bwd": [_CFG] + [P] * 13 + [ctypes.c_size_t, P],
+    "moe_dispatch_bwd": [_CFG] + [P] * 6,
     "moe_device_status": [P, ctypes.POINTER(ctypes.c_int32)],
     "moe_set_wait_limit_ns": [ctypes.c_uint64],
     "moe_set_gemm_pairs": [ctypes.c_int],
@@ -208,12 +208,11 @@ def moe_expert_ffn_bwd(cfg, x_perm, offsets, w1, w2, h_gu, act, dy_perm, dh, dx_
 
 
 def moe_route_bwd(cfg, x, w_router, probs, topk_idx, topk_w, dtopk_w, aux_coef, party_offsets,
-                  dlogits, dw_router, dbias, workspace, workspace_bytes, stream=None):
+                  dlogits, dw_router, dbias, dx_router, workspace, workspace_bytes, stream=None):
     _call("moe_route_bwd", cfg, x, w_router, probs, topk_idx, topk_w, dtopk_w, aux_coef,
-          party_offsets, dlogits, dw_router, dbias, workspace, int(workspace_bytes), stream=stream)
-
-
-def moe_dispatch_bwd(cfg, dx_perm, slot_of, dlogits, w_router, party_offsets, dx_sh, dx,
-                     stream=None):
-    _call("moe_dispatch_bwd", cfg, dx_perm, slot_of, dlogits, w_router, party_offsets, dx_sh, dx,
+          party_offsets, dlogits, dw_router, dbias, dx_router, workspace, int(workspace_bytes),
           stream=stream)
+
+
+def moe_dispatch_bwd(cfg, dx_perm, slot_of, dx_router, dx_sh, dx, stream=None):
+    _call("moe_dispatch_bwd", cfg, dx_perm, slot_of, dx_router, dx_sh, dx, stream=stream)

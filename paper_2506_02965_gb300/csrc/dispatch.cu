@@ -118,10 +118,19 @@ __global__ void __launch_bounds__(256) gather_kernel(const T* __restrict__ x,
         return;
     }
     constexpr int VN = Vec<T>::N;
+    constexpr int U = 4;  // vectors per lane in flight
     const int nv = d / VN;
     const T* src = x + t * d;
     T* dst = x_perm + r * d;
-    for (int v = lane; v < nv; v += 32) Vec<T>::raw_store(dst + v * VN, Vec<T>::raw_load(src + v * VN));
+    for (int v0 = lane; v0 < nv; v0 += 32 * U) {
+        uint4 buf[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u)
+            if (v0 + 32 * u < nv) buf[u] = Vec<T>::raw_load(src + (v0 + 32 * u) * VN);
+#pragma unroll
+        for (int u = 0; u < U; ++u)
+            if (v0 + 32 * u < nv) Vec<T>::raw_store(dst + (v0 + 32 * u) * VN, buf[u]);
+    }
 }
 
 // out[t] = sum_j w[t,j] * y_perm[slot_of[t,j]] (+ sum_s y_sh[s,t]); fp32 accumulation.
@@ -257,134 +266,70 @@ __global__ void __launch_bounds__(256, 3) combine_bwd_kernel(const T* __restrict
     }
 }
 
-// dx[t] = sum_j dx_perm[slot(t,j)] + sum_e dlogits[t,e] W_r[p(t)][e] + sum_s dx_sh[s,t].
-// A block takes UR_TOK tokens of one party and a slab of 64 * VN columns; each thread
-// owns VN columns of UR_TOK / 4 tokens. The slot lookups and permuted rows of the first
-// two picks are requested first; while they are in flight the party's router rows for
-// the slab and the tokens' dlogits are staged in shared memory and the router term is
-// accumulated.
-constexpr int UR_TOK = 16;
-constexpr int UR_PRE = 2;  // picks whose rows are loaded before the router term
-
-template <typename T>
-__global__ void __launch_bounds__(256) unpermute_reduce_kernel(
+// dx[t] = sum_j dx_perm[slot(t,j)] + dx_router[t] + sum_s dx_sh[s,t]; fp32 accumulation.
+// One warp per token; every lane issues the loads of up to UB vectors of all k rows (and
+// of the router's row) before it uses any of them.
+template <typename T, int KMAX>
+__global__ void __launch_bounds__(256, 3) unpermute_reduce_kernel(
     const T* __restrict__ dx_perm, const int32_t* __restrict__ slot_of,
-    const float* __restrict__ dz, const T* __restrict__ wr, const int32_t* __restrict__ po, int P,
-    const T* __restrict__ dx_sh, int S, int64_t Tn, int d, int E, int k, T* dx) {
+    const T* __restrict__ dx_router, const T* __restrict__ dx_sh, int S, int64_t Tn, int d, int k,
+    T* dx) {
     pdl_begin();
+    const int lane = threadIdx.x & 31;
+    const int64_t t = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    if (t >= Tn) return;
     constexpr int VN = Vec<T>::N;
-    constexpr int SLAB = 64 * VN;
-    constexpr int TPT = UR_TOK / 4;  // tokens per thread
-    extern __shared__ __align__(16) unsigned char ur_smem[];
-    float* s_dz = reinterpret_cast<float*>(ur_smem);                  // [UR_TOK][E]
-    T* s_w = reinterpret_cast<T*>(ur_smem + UR_TOK * 64 * sizeof(float));  // [E][SLAB]
-    // tile -> (party, first token)
-    int64_t ti = blockIdx.x, t0 = -1, tend = 0;
-    int party = 0;
-    for (int p = 0; p < P; ++p) {
-        const int64_t a = po ? po[p] : 0, b = po ? po[p + 1] : Tn;
-        const int64_t nt = (b - a + UR_TOK - 1) / UR_TOK;
-        if (ti < nt) { party = p; t0 = a + ti * UR_TOK; tend = b; break; }
-        ti -= nt;
-    }
-    if (t0 < 0) return;
-    const int n = (int)min64(UR_TOK, tend - t0);
-    const int64_t c0 = (int64_t)blockIdx.y * SLAB;
-    const int ncols = (int)min64(SLAB, d - c0);
-    const int cv = threadIdx.x & 63;  // column vector inside the slab
-    const int tg = threadIdx.x >> 6;  // token group
-    const bool active = cv * VN < ncols;
-    const int64_t col = c0 + cv * VN;
-    // slot of pick j of this thread's tokens (-1: no token, or a bad slot, recorded)
-    auto slots_of = [&](int j, int32_t* slot) {
+    constexpr int UB = KMAX <= 2 ? 4 : KMAX <= 4 ? 2 : 1;  // vectors per lane in flight
+    int32_t slot[KMAX];
 #pragma unroll
-        for (int i = 0; i < TPT; ++i) {
-            const int tt = tg * TPT + i;
-            slot[i] = (active && tt < n) ? slot_of[(t0 + tt) * k + j] : -1;
-            if (active && tt < n && (slot[i] < 0 || (int64_t)slot[i] >= Tn * k)) {
-                if (cv == 0) record_status(MOE_ERR_DEVICE_CHECK);
-                slot[i] = -1;
+    for (int j = 0; j < KMAX; ++j) {
+        slot[j] = j < k ? slot_of[t * k + j] : -1;
+        if (j < k && (slot[j] < 0 || (int64_t)slot[j] >= Tn * k)) {  // bad table: skip the row
+            if (lane == 0) record_status(MOE_ERR_DEVICE_CHECK);
+            slot[j] = -1;
+        }
+    }
+    const int nv = d / VN;
+    for (int v0 = lane; v0 < nv; v0 += 32 * UB) {
+        uint4 raw[UB][KMAX], rr[UB];
+#pragma unroll
+        for (int u = 0; u < UB; ++u) {
+            const int v = v0 + 32 * u;
+            if (v < nv) {
+#pragma unroll
+                for (int j = 0; j < KMAX; ++j)
+                    if (slot[j] >= 0) raw[u][j] = Vec<T>::raw_load(dx_perm + (int64_t)slot[j] * d + v * VN);
+                if (dx_router) rr[u] = Vec<T>::raw_load(dx_router + t * d + v * VN);
             }
         }
-    };
-    int32_t pslot[UR_PRE][TPT];
-    uint4 praw[UR_PRE][TPT];
 #pragma unroll
-    for (int j = 0; j < UR_PRE; ++j) {
-        if (j < k) {
-            slots_of(j, pslot[j]);
-        } else {
+        for (int u = 0; u < UB; ++u) {
+            const int v = v0 + 32 * u;
+            if (v >= nv) break;
+            float acc[VN];
+            if (dx_router) {
+                unpack_vec<T>(rr[u], acc);
+            } else {
 #pragma unroll
-            for (int i = 0; i < TPT; ++i) pslot[j][i] = -1;
-        }
-    }
+                for (int q = 0; q < VN; ++q) acc[q] = 0.f;
+            }
 #pragma unroll
-    for (int j = 0; j < UR_PRE; ++j)
+            for (int j = 0; j < KMAX; ++j) {
+                if (slot[j] >= 0) {
+                    float g[VN];
+                    unpack_vec<T>(raw[u][j], g);
 #pragma unroll
-        for (int i = 0; i < TPT; ++i)
-            if (pslot[j][i] >= 0) praw[j][i] = Vec<T>::raw_load(dx_perm + (int64_t)pslot[j][i] * d + col);
-    // router term: stage dlogits and the party's router rows for this slab
-    const T* W = wr + (int64_t)party * E * d;
-    for (int i = threadIdx.x; i < UR_TOK * E; i += blockDim.x) {
-        const int tt = i / E, e = i % E;
-        s_dz[i] = tt < n ? dz[(t0 + tt) * E + e] : 0.f;
-    }
-    for (int i = threadIdx.x; i < E * (SLAB / VN); i += blockDim.x) {
-        const int e = i / (SLAB / VN), v = i % (SLAB / VN);
-        if (v * VN < ncols) Vec<T>::raw_store(s_w + e * SLAB + v * VN, Vec<T>::raw_load(W + (int64_t)e * d + c0 + v * VN));
-    }
-    __syncthreads();
-    if (!active) return;
-    float acc[TPT][VN];
-#pragma unroll
-    for (int i = 0; i < TPT; ++i)
-#pragma unroll
-        for (int q = 0; q < VN; ++q) acc[i][q] = 0.f;
-    for (int e = 0; e < E; ++e) {
-        float wv[VN];
-        Vec<T>::load(s_w + e * SLAB + cv * VN, wv);
-#pragma unroll
-        for (int i = 0; i < TPT; ++i) {
-            const float zz = s_dz[(tg * TPT + i) * E + e];
-#pragma unroll
-            for (int q = 0; q < VN; ++q) acc[i][q] = fmaf(zz, wv[q], acc[i][q]);
-        }
-    }
-    auto add_rows = [&](const int32_t* slot, const uint4* raw) {
-#pragma unroll
-        for (int i = 0; i < TPT; ++i) {
-            if (slot[i] >= 0) {
+                    for (int q = 0; q < VN; ++q) acc[q] += g[q];
+                }
+            }
+            for (int s2 = 0; s2 < S; ++s2) {
                 float g[VN];
-                unpack_vec<T>(raw[i], g);
+                Vec<T>::load(dx_sh + ((int64_t)s2 * Tn + t) * d + v * VN, g);
 #pragma unroll
-                for (int q = 0; q < VN; ++q) acc[i][q] += g[q];
+                for (int q = 0; q < VN; ++q) acc[q] += g[q];
             }
+            Vec<T>::store(dx + t * d + v * VN, acc);
         }
-    };
-#pragma unroll
-    for (int j = 0; j < UR_PRE; ++j) add_rows(pslot[j], praw[j]);
-    // remaining picks, one at a time: the slot lookups, then the rows, in flight together
-    for (int j = UR_PRE; j < k; ++j) {
-        int32_t slot[TPT];
-        slots_of(j, slot);
-        uint4 raw[TPT];
-#pragma unroll
-        for (int i = 0; i < TPT; ++i)
-            if (slot[i] >= 0) raw[i] = Vec<T>::raw_load(dx_perm + (int64_t)slot[i] * d + col);
-        add_rows(slot, raw);
-    }
-#pragma unroll
-    for (int i = 0; i < TPT; ++i) {
-        const int tt = tg * TPT + i;
-        if (tt >= n) break;
-        const int64_t t = t0 + tt;
-        for (int s2 = 0; s2 < S; ++s2) {
-            float g[VN];
-            Vec<T>::load(dx_sh + ((int64_t)s2 * Tn + t) * d + col, g);
-#pragma unroll
-            for (int q = 0; q < VN; ++q) acc[i][q] += g[q];
-        }
-        Vec<T>::store(dx + t * d + col, acc[i]);
     }
 }
 
@@ -462,40 +407,24 @@ cudaError_t launch_combine_bwd(const void* dout, const void* y_perm, const float
 }
 
 cudaError_t launch_unpermute_reduce(const void* dx_perm, const int32_t* slot_of,
-                                    const float* dlogits, const void* w_router,
-                                    const int32_t* po, int P, const void* dx_sh, int S, int64_t T,
-                                    int d, int E, int k, bool bf16, void* dx, cudaStream_t s) {
+                                    const void* dx_router, const void* dx_sh, int S, int64_t T,
+                                    int d, int k, bool bf16, void* dx, cudaStream_t s) {
     if (T == 0) return cudaSuccess;
-    const unsigned tiles = (unsigned)((T + UR_TOK - 1) / UR_TOK + P);
-    const int VN = bf16 ? 8 : 4;
-    const int slab = 64 * VN;
-    dim3 grid(tiles, (d + slab - 1) / slab);
-    const size_t smem = UR_TOK * 64 * sizeof(float) + (size_t)E * slab * (bf16 ? 2 : 4);
+    const unsigned blocks = (unsigned)((T + 7) / 8);
+#define MOE_UR(TT, KM)                                                                            \
+    (void)launch_pdl(unpermute_reduce_kernel<TT, KM>, dim3(blocks), dim3(256), 0, s,              \
+                     (const TT*)dx_perm, slot_of, (const TT*)dx_router, (const TT*)dx_sh, S, T, d, \
+                     k, (TT*)dx)
     if (bf16) {
-        static bool attr = false;
-        if (!attr) {
-            cudaError_t e = cudaFuncSetAttribute(unpermute_reduce_kernel<__nv_bfloat16>,
-                                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 (int)(UR_TOK * 64 * 4 + 64 * 512 * 2));
-            if (e != cudaSuccess) return e;
-            attr = true;
-        }
-        (void)launch_pdl(unpermute_reduce_kernel<__nv_bfloat16>, dim3(grid), dim3(256), smem, s, 
-            (const __nv_bfloat16*)dx_perm, slot_of, dlogits, (const __nv_bfloat16*)w_router, po, P,
-            (const __nv_bfloat16*)dx_sh, S, T, d, E, k, (__nv_bfloat16*)dx);
+        if (k <= 2) MOE_UR(__nv_bfloat16, 2);
+        else if (k <= 4) MOE_UR(__nv_bfloat16, 4);
+        else MOE_UR(__nv_bfloat16, 8);
     } else {
-        static bool attr = false;
-        if (!attr) {
-            cudaError_t e = cudaFuncSetAttribute(unpermute_reduce_kernel<float>,
-                                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 (int)(UR_TOK * 64 * 4 + 64 * 256 * 4));
-            if (e != cudaSuccess) return e;
-            attr = true;
-        }
-        (void)launch_pdl(unpermute_reduce_kernel<float>, dim3(grid), dim3(256), smem, s, 
-            (const float*)dx_perm, slot_of, dlogits, (const float*)w_router, po, P,
-            (const float*)dx_sh, S, T, d, E, k, (float*)dx);
+        if (k <= 2) MOE_UR(float, 2);
+        else if (k <= 4) MOE_UR(float, 4);
+        else MOE_UR(float, 8);
     }
+#undef MOE_UR
     return cudaGetLastError();
 }
 

@@ -873,6 +873,26 @@ __global__ void __launch_bounds__(THREADS, 1)
                     }
                 } else if constexpr (EPI == EPI_ROUTE) {
                     route_epilogue<BN>(p, ti, m, valid, tbase, route_hist);
+                } else if constexpr (EPI == EPI_DWR) {
+                    // one token chunk's partial router gradient: accumulator row m is model
+                    // column m, column e is expert e; stored transposed, fp32, part[g][e][m]
+                    // (a warp's 32 rows are 32 consecutive floats of one expert row)
+                    float* part = (float*)p.out0 + (int64_t)ti.g * p.E * p.Mout + m;
+#pragma unroll 1
+                    for (int c = 0; c < BN; c += 32) {
+                        float v[32];
+                        if (ti.k_iters > 0) {
+                            tmem_ld32(tbase + c, v);
+                        } else {
+#pragma unroll
+                            for (int i = 0; i < 32; ++i) v[i] = 0.f;
+                        }
+                        if (valid) {
+#pragma unroll
+                            for (int i = 0; i < 32; ++i)
+                                if (c + i < p.E) part[(int64_t)(c + i) * p.Mout] = v[i];
+                        }
+                    }
                 } else {
                     __nv_bfloat16* out;
                     if (VAR_K)
@@ -1119,9 +1139,9 @@ cudaError_t launch_gemm_m(const GemmMArgs& g, bool bf16, cudaStream_t s) {
         if (!make_map(&mb, g.b, g.K, (int64_t)g.G * g.N, 128)) return cudaErrorInvalidValue;
         return launch<128, false, false, EPI_STORE>(ma, mb, mo0, mo0, p, mt_ub * (g.N / 128), s);
     }
-    // MN-major B: weights stored [G*K, N]
-    p.b_group_rows = g.K;
-    if (!make_map(&mb, g.b, g.N, (int64_t)g.G * g.K, 64)) return cudaErrorInvalidValue;
+    // MN-major B: weights stored [G*K, N] (or [G*b_rows, N])
+    p.b_group_rows = g.b_rows ? g.b_rows : g.K;
+    if (!make_map(&mb, g.b, g.N, (int64_t)g.G * p.b_group_rows, 64)) return cudaErrorInvalidValue;
     if (g.epi == EPI_SWIGLU_BWD) {
         p.F = g.N;
         if (!make_map(&mo0, g.out0, 2 * (int64_t)g.N, o_rows, 0, true)) return cudaErrorInvalidValue;
@@ -1162,8 +1182,13 @@ cudaError_t launch_gemm_k(const GemmKArgs& g, bool bf16, cudaStream_t s) {
     CUtensorMap ma, mb, mo;
     if (!make_map(&ma, g.a, g.M, rows_a, 64)) return cudaErrorInvalidValue;
     if (!make_map(&mb, g.b, g.N, rows_b, 64)) return cudaErrorInvalidValue;
-    if (!make_map(&mo, g.out, g.N, (int64_t)g.G * g.M, 0, true)) return cudaErrorInvalidValue;
     const int64_t tiles = (int64_t)g.G * (g.M / BM);
+    if (g.epi == EPI_DWR) {  // fp32 partials, N = 64 (experts, zero-padded)
+        if (g.N != 64 || g.M % BM) return cudaErrorInvalidValue;
+        p.E = g.E;
+        return launch<64, true, true, EPI_DWR>(ma, mb, ma, ma, p, tiles, s);
+    }
+    if (!make_map(&mo, g.out, g.N, (int64_t)g.G * g.M, 0, true)) return cudaErrorInvalidValue;
     if (g.N % 256 == 0) return launch<256, true, true, EPI_STORE>(ma, mb, mo, mo, p, tiles * (g.N / 256), s);
     return launch<128, true, true, EPI_STORE>(ma, mb, mo, mo, p, tiles * (g.N / 128), s);
 }

@@ -549,13 +549,16 @@ moe_status moe_route_bwd(const moe_config* cfg, const void* x, const void* w_rou
                          const float* probs, const int32_t* topk_idx, const float* topk_w,
                          const float* dtopk_w, const float* aux_coef,
                          const int32_t* party_offsets, float* dlogits, void* dw_router,
-                         float* dbias, void* workspace, size_t workspace_bytes,
-                         moe_stream_t stream) {
+                         float* dbias, void* dx_router, void* workspace,
+                         size_t workspace_bytes, moe_stream_t stream) {
     moe_status st = check_cfg(cfg);
     if (st) return st;
     if ((st = check_parties(cfg, party_offsets))) return st;
-    (void)w_router;
     REQUIRE_VEC(dw_router);
+    if (dx_router && cfg->T > 0) {
+        REQUIRE_VEC(dx_router);
+        REQUIRE_VEC(w_router);
+    }
     if (cfg->T > 0) {
         REQUIRE_VEC(x);
         REQUIRE(probs);
@@ -585,27 +588,25 @@ moe_status moe_route_bwd(const moe_config* cfg, const void* x, const void* w_rou
     a.dlogits = dlogits;
     a.dw_router = dw_router;
     a.dbias = dbias;
+    a.w_router = w_router;
+    a.dx_router = dx_router;
     return cuda_status(launch_route_bwd(a, cfg->dtype == MOE_BF16, workspace, (cudaStream_t)stream),
                        "moe_route_bwd");
 }
 
 moe_status moe_dispatch_bwd(const moe_config* cfg, const void* dx_perm, const int32_t* slot_of,
-                            const float* dlogits, const void* w_router,
-                            const int32_t* party_offsets, const void* dx_sh, void* dx,
+                            const void* dx_router, const void* dx_sh, void* dx,
                             moe_stream_t stream) {
     moe_status st = check_cfg(cfg);
     if (st) return st;
-    if ((st = check_parties(cfg, party_offsets))) return st;
     if (cfg->T == 0) return MOE_OK;
     REQUIRE_VEC(dx_perm);
     REQUIRE(slot_of);
-    REQUIRE(dlogits);
-    REQUIRE_VEC(w_router);
+    if (dx_router) REQUIRE_VEC(dx_router);
     REQUIRE_VEC(dx);
     if (cfg->n_shared) REQUIRE_VEC(dx_sh);
-    return cuda_status(launch_unpermute_reduce(dx_perm, slot_of, dlogits, w_router, party_offsets,
-                                               cfg->n_parties, dx_sh, cfg->n_shared, cfg->T,
-                                               cfg->d_model, cfg->n_experts, cfg->top_k,
+    return cuda_status(launch_unpermute_reduce(dx_perm, slot_of, dx_router, dx_sh, cfg->n_shared,
+                                               cfg->T, cfg->d_model, cfg->top_k,
                                                cfg->dtype == MOE_BF16, dx, (cudaStream_t)stream),
                        "moe_dispatch_bwd");
 }

@@ -37,6 +37,8 @@ struct RouteBwdArgs {
     float* dlogits;
     void* dw_router;
     float* dbias;
+    const void* w_router;  // [P,E,d]
+    void* dx_router;       // [T,d] or null
 };
 
 cudaError_t launch_route(const RouteArgs& a, bool bf16, bool from_logits, cudaStream_t s);
@@ -61,9 +63,8 @@ cudaError_t launch_combine_bwd(const void* dout, const void* y_perm, const float
                                const int32_t* slot_of, int64_t T, int d, int k, bool bf16,
                                void* dy_perm, float* dtopk_w, cudaStream_t s);
 cudaError_t launch_unpermute_reduce(const void* dx_perm, const int32_t* slot_of,
-                                    const float* dlogits, const void* w_router,
-                                    const int32_t* po, int P, const void* dx_sh, int S, int64_t T,
-                                    int d, int E, int k, bool bf16, void* dx, cudaStream_t s);
+                                    const void* dx_router, const void* dx_sh, int S, int64_t T,
+                                    int d, int k, bool bf16, void* dx, cudaStream_t s);
 cudaError_t dispatch_status(cudaStream_t s, int* code);
 // dispatch with its per-chunk counts in a fixed device array (no workspace argument)
 constexpr int64_t kNoAllocScratchInts = 1 << 16;  // 256 KiB of int32 chunk counts
@@ -73,7 +74,7 @@ cudaError_t launch_dispatch_noalloc(const int32_t* topk_idx, const void* x, int6
                                     int32_t* token_of, void* x_perm, cudaStream_t s);
 
 // grouped GEMMs -------------------------------------------------------------------------
-enum EpiKind { EPI_SWIGLU_FWD = 0, EPI_STORE = 1, EPI_SWIGLU_BWD = 2, EPI_ROUTE = 3 };
+enum EpiKind { EPI_SWIGLU_FWD = 0, EPI_STORE = 1, EPI_SWIGLU_BWD = 2, EPI_ROUTE = 3, EPI_DWR = 4 };
 
 // How the groups (experts) of a grouped GEMM are laid out along the rows that vary:
 //  OFFSETS: group g owns rows [offsets[g], offsets[g+1]) of A / out (M-variable) or of
@@ -99,6 +100,8 @@ struct GemmMArgs {
     int64_t b_group_elems;
     bool b_kmajor;
     int N, K;
+    int b_rows;  // MN-major B: rows of one group's [K, N] view when they are fewer than K
+                 // (the rows past them multiply zero columns of A); 0 means K
     int epi;
     // EPI_SWIGLU_FWD: out0 = h_gu [rows, 2F] (G at cols [0,F), U at [F,2F)),
     //                 out1 = act [rows, F]; N = 2F (B holds gate rows then up rows).
@@ -118,6 +121,10 @@ struct GemmKArgs {
     const void* b;
     int M, N;
     void* out;
+    // EPI_STORE: out = dtype C as above. EPI_DWR (bf16 only, N = 64): out = fp32 partials
+    // stored transposed, out + (g*E + e)*M + m = C_g[m, e] for e < E.
+    int epi = EPI_STORE;
+    int E = 0;
 };
 
 cudaError_t launch_gemm_m(const GemmMArgs& g, bool bf16, cudaStream_t s);

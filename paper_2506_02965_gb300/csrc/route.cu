@@ -5,6 +5,8 @@
 
 #include <cooperative_groups.h>
 
+#include <algorithm>
+
 #include "moe_common.cuh"
 #include "moe_internal.h"
 
@@ -250,15 +252,27 @@ __device__ __forceinline__ bool chunk_of(int64_t ci, const int32_t* po, int P, i
 }
 
 // dlogits, one warp per token (Alg. 7 backward with the picks held fixed); lane l
-// holds experts l and l + 32.
+// holds experts l and l + 32. For the tensor-core router gradients it also writes
+// dz16 [T, 64], dlogits rounded to bf16 with zero columns past E, and (block 0) the
+// token chunks of the chunked dW_r contraction: chunk_off[c] = first token of chunk c,
+// the chunks of CH tokens of each party in order, then empty chunks up to nchunk.
 __global__ void __launch_bounds__(256) dlogits_kernel(
     const float* __restrict__ probs, const int32_t* __restrict__ topk_idx,
     const float* __restrict__ topk_w, const float* __restrict__ dtopk_w,
     const float* __restrict__ aux_coef, const int32_t* __restrict__ po, int P, int64_t Tn, int E,
-    int k, int normalize, float* dlogits) {
+    int k, int normalize, float* dlogits, __nv_bfloat16* dz16, int32_t* chunk_off, int CH,
+    int nchunk) {
     pdl_begin();
     const int lane = threadIdx.x & 31;
     const int64_t t = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    if (chunk_off && blockIdx.x == 0 && threadIdx.x == 0) {
+        int c = 0;
+        for (int q = 0; q < P; ++q) {
+            const int64_t a = po ? po[q] : 0, b = po ? po[q + 1] : Tn;
+            for (int64_t r = a; r < b && c < nchunk; r += CH) chunk_off[c++] = (int32_t)r;
+        }
+        for (; c <= nchunk; ++c) chunk_off[c] = (int32_t)Tn;
+    }
     if (t >= Tn) return;
     const int party = party_of(po, P, t);
     const int e0 = lane, e1 = lane + 32;
@@ -283,8 +297,30 @@ __global__ void __launch_bounds__(256) dlogits_kernel(
         if (e == e1) dp1 += g;
     }
     const float dot = warp_sum(dp0 * p0 + dp1 * p1);
-    if (e0 < E) dlogits[t * E + e0] = p0 * (dp0 - dot);
-    if (e1 < E) dlogits[t * E + e1] = p1 * (dp1 - dot);
+    const float z0 = p0 * (dp0 - dot), z1 = p1 * (dp1 - dot);
+    if (e0 < E) dlogits[t * E + e0] = z0;
+    if (e1 < E) dlogits[t * E + e1] = z1;
+    if (dz16) {
+        dz16[t * 64 + e0] = __float2bfloat16_rn(e0 < E ? z0 : 0.f);
+        dz16[t * 64 + e1] = __float2bfloat16_rn(e1 < E ? z1 : 0.f);
+    }
+}
+
+// dbias partial of one token chunk: part_db[c][e] = sum of dlogits[t][e] over the chunk,
+// four token strides summed in a fixed order.
+__global__ void __launch_bounds__(256) chunk_db_kernel(const float* __restrict__ dz,
+                                                      const int32_t* __restrict__ chunk_off, int E,
+                                                      float* part_db) {
+    pdl_begin();
+    __shared__ float s_part[4][64];
+    const int c = blockIdx.x, e = threadIdx.x & 63, g = threadIdx.x >> 6;
+    const int64_t a = chunk_off[c], b = chunk_off[c + 1];
+    float acc = 0.f;
+    if (e < E)
+        for (int64_t t = a + g; t < b; t += 4) acc += dz[t * E + e];
+    s_part[g][e] = acc;
+    __syncthreads();
+    if (g == 0 && e < E) part_db[(int64_t)c * E + e] = ((s_part[0][e] + s_part[1][e]) + s_part[2][e]) + s_part[3][e];
 }
 
 // Partial dW_r = dlogits^T x and db over one chunk of RB_CH tokens of one party, for
@@ -379,7 +415,8 @@ constexpr int RR_OUT = 32, RR_GRP = 8;
 template <typename T>
 __global__ void __launch_bounds__(RR_OUT * RR_GRP) route_bwd_reduce_kernel(
     const float* __restrict__ part_dw, const float* __restrict__ part_db,
-    const int32_t* __restrict__ po, int P, int64_t Tn, int d, int E, T* dw_router, float* dbias) {
+    const int32_t* __restrict__ po, int P, int64_t Tn, int d, int E, int CH, T* dw_router,
+    float* dbias) {
     pdl_begin();
     __shared__ float s_sum[RR_GRP][RR_OUT];
     const int o = threadIdx.x % RR_OUT, g = threadIdx.x / RR_OUT;
@@ -389,7 +426,7 @@ __global__ void __launch_bounds__(RR_OUT * RR_GRP) route_bwd_reduce_kernel(
         int64_t base = 0;
         for (int q = 0; q < P; ++q) {
             int64_t a = po ? po[q] : 0, b = po ? po[q + 1] : Tn;
-            int64_t nc = (b - a + RB_CH - 1) / RB_CH;
+            int64_t nc = (b - a + CH - 1) / CH;
             if (q == p) { *first = base; *cnt = nc; return; }
             base += nc;
         }
@@ -476,20 +513,50 @@ cudaError_t launch_aux_loss(const float* probs, const int32_t* counts, const int
     return cudaGetLastError();
 }
 
-size_t route_bwd_workspace(int64_t T, int P, int E, int d) {
-    const int64_t nch = (T + RB_CH - 1) / RB_CH + P;
-    return (size_t)nch * E * d * sizeof(float) + (size_t)nch * E * sizeof(float) + 256;
+// Workspace of the router backward. CUDA-core path (fp32): per-chunk partials of
+// RB_CH tokens. Tensor-core path (bf16): per-chunk fp32 partials of dW_r and dbias, the
+// chunk table and dz16 [T, 64] (dlogits in bf16, the A operand of dx_router = dz W_r and
+// the B operand of dW_r^T = x^T dz).
+static size_t align256(size_t n) { return (n + 255) / 256 * 256; }
+struct RbTcLayout {
+    int64_t C, nchunk;
+    size_t dw, db, off, dz, total;
+};
+// Tokens per chunk of the chunked dW_r contraction: about 256 tiles of 128 model columns
+// in all, at most 128 - P chunks (the grouped GEMM's group limit), a multiple of 64.
+static RbTcLayout rb_tc_layout(int64_t T, int P, int E, int d) {
+    RbTcLayout L;
+    const int64_t mt = std::max(1, d / 128);
+    int64_t C = (T * mt + 255) / 256;
+    C = std::max<int64_t>(C, (T + (128 - P) - 1) / (128 - P));
+    C = std::max<int64_t>(C, 64);
+    L.C = (C + 63) / 64 * 64;
+    L.nchunk = (T + L.C - 1) / L.C + P;
+    L.dw = 0;
+    L.db = align256((size_t)L.nchunk * E * d * sizeof(float));
+    L.off = align256(L.db + (size_t)L.nchunk * E * sizeof(float));
+    L.dz = align256(L.off + (size_t)(L.nchunk + 1) * sizeof(int32_t));
+    L.total = L.dz + (size_t)T * 64 * 2 + 256;
+    return L;
 }
 
-template <typename T>
-static cudaError_t launch_route_bwd_t(const RouteBwdArgs& a, void* ws, cudaStream_t s) {
+size_t route_bwd_workspace(int64_t T, int P, int E, int d) {
+    const int64_t nch = (T + RB_CH - 1) / RB_CH + P;
+    const size_t simt = (size_t)nch * E * d * sizeof(float) + (size_t)nch * E * sizeof(float) + 256;
+    return std::max(simt, rb_tc_layout(T, P, E, d).total);
+}
+
+// fp32: dlogits, CUDA-core partials and reduce, dx_router on the CUDA-core GEMM
+static cudaError_t launch_route_bwd_simt(const RouteBwdArgs& a, void* ws, cudaStream_t s) {
+    using T = float;
     const int64_t nch = (a.T + RB_CH - 1) / RB_CH + a.P;
     float* part_dw = (float*)ws;
     float* part_db = part_dw + nch * a.E * a.d;
     if (a.T > 0) {
         const unsigned blocks = (unsigned)((a.T + 7) / 8);
-        (void)launch_pdl(dlogits_kernel, dim3(blocks), dim3(256), 0, s, a.probs, a.topk_idx, a.topk_w, a.dtopk_w, a.aux_coef,
-                                              a.po, a.P, a.T, a.E, a.k, a.normalize, a.dlogits);
+        (void)launch_pdl(dlogits_kernel, dim3(blocks), dim3(256), 0, s, a.probs, a.topk_idx, a.topk_w,
+                         a.dtopk_w, a.aux_coef, a.po, a.P, a.T, a.E, a.k, a.normalize, a.dlogits,
+                         (__nv_bfloat16*)nullptr, (int32_t*)nullptr, 0, 0);
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
     }
@@ -503,18 +570,91 @@ static cudaError_t launch_route_bwd_t(const RouteBwdArgs& a, void* ws, cudaStrea
         if (e != cudaSuccess) return e;
         attr = true;
     }
-    (void)launch_pdl(route_bwd_partial_kernel<T>, dim3(grid), dim3(2 * RB_HALF), smem, s, (const T*)a.x, a.dlogits, a.po,
-                                                                a.P, a.T, a.d, a.E, part_dw, part_db);
+    (void)launch_pdl(route_bwd_partial_kernel<T>, dim3(grid), dim3(2 * RB_HALF), smem, s, (const T*)a.x,
+                     a.dlogits, a.po, a.P, a.T, a.d, a.E, part_dw, part_db);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     const int64_t total = (int64_t)a.P * a.E * a.d;
-    (void)launch_pdl(route_bwd_reduce_kernel<T>, dim3((unsigned)((total + RR_OUT - 1) / RR_OUT)), dim3(RR_OUT * RR_GRP), 0, s, 
-        part_dw, part_db, a.po, a.P, a.T, a.d, a.E, (T*)a.dw_router, a.dbias);
-    return cudaGetLastError();
+    (void)launch_pdl(route_bwd_reduce_kernel<T>, dim3((unsigned)((total + RR_OUT - 1) / RR_OUT)),
+                     dim3(RR_OUT * RR_GRP), 0, s, part_dw, part_db, a.po, a.P, a.T, a.d, a.E, RB_CH,
+                     (T*)a.dw_router, a.dbias);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if (a.dx_router && a.T > 0) {  // dx_router[t] = dlogits[t] W_r[p(t)], K = E
+        GemmMArgs m{};
+        m.G = a.po ? a.P : 1;
+        m.rows = GroupRows{a.po, (int)a.T, 0, 0, 0};
+        m.a = a.dlogits;
+        m.b = a.w_router;
+        m.b_group_elems = (int64_t)a.E * a.d;
+        m.b_kmajor = false;
+        m.N = a.d;
+        m.K = a.E;
+        m.epi = EPI_STORE;
+        m.out0 = a.dx_router;
+        return launch_gemm_m_simt(m, s);
+    }
+    return cudaSuccess;
+}
+
+// bf16: both products on the tensor cores.
+//   dW_r[p]^T = sum over the chunks c of party p of x_c^T dz_c (K-variable grouped GEMM,
+//               one group per chunk, fp32 partials), reduced over chunks in order;
+//   dx_router = dz W_r[p(t)] (M-variable grouped GEMM over parties, K = 64 padded).
+// dz is rounded to bf16 for both (the operands of every bf16 contraction are bf16).
+static cudaError_t launch_route_bwd_tc(const RouteBwdArgs& a, void* ws, cudaStream_t s) {
+    const RbTcLayout Lw = rb_tc_layout(a.T, a.P, a.E, a.d);
+    uint8_t* base = (uint8_t*)ws;
+    float* part_dw = (float*)(base + Lw.dw);
+    float* part_db = (float*)(base + Lw.db);
+    int32_t* chunk_off = (int32_t*)(base + Lw.off);
+    __nv_bfloat16* dz16 = (__nv_bfloat16*)(base + Lw.dz);
+    cudaError_t e;
+    if (a.T > 0) {
+        const unsigned blocks = (unsigned)((a.T + 7) / 8);
+        (void)launch_pdl(dlogits_kernel, dim3(blocks), dim3(256), 0, s, a.probs, a.topk_idx, a.topk_w,
+                         a.dtopk_w, a.aux_coef, a.po, a.P, a.T, a.E, a.k, a.normalize, a.dlogits, dz16,
+                         chunk_off, (int)Lw.C, (int)Lw.nchunk);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+        (void)launch_pdl(chunk_db_kernel, dim3((unsigned)Lw.nchunk), dim3(256), 0, s,
+                         (const float*)a.dlogits, (const int32_t*)chunk_off, a.E, part_db);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+        GemmKArgs g{};
+        g.G = (int)Lw.nchunk;
+        g.rows = GroupRows{chunk_off, (int)a.T, 0, 0, 0};
+        g.a = a.x;
+        g.b = dz16;
+        g.M = a.d;
+        g.N = 64;
+        g.out = part_dw;
+        g.epi = EPI_DWR;
+        g.E = a.E;
+        if ((e = launch_gemm_k(g, true, s)) != cudaSuccess) return e;
+    }
+    const int64_t total = (int64_t)a.P * a.E * a.d;
+    (void)launch_pdl(route_bwd_reduce_kernel<__nv_bfloat16>, dim3((unsigned)((total + RR_OUT - 1) / RR_OUT)),
+                     dim3(RR_OUT * RR_GRP), 0, s, (const float*)part_dw, (const float*)part_db, a.po, a.P,
+                     a.T, a.d, a.E, (int)Lw.C, (__nv_bfloat16*)a.dw_router, a.dbias);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if (a.dx_router && a.T > 0) {
+        GemmMArgs m{};
+        m.G = a.po ? a.P : 1;
+        m.rows = GroupRows{a.po, (int)a.T, 0, 0, 0};
+        m.a = dz16;
+        m.b = a.w_router;
+        m.b_group_elems = (int64_t)a.E * a.d;
+        m.b_kmajor = false;
+        m.N = a.d;
+        m.K = 64;
+        m.b_rows = a.E;
+        m.epi = EPI_STORE;
+        m.out0 = a.dx_router;
+        return launch_gemm_m(m, true, s);
+    }
+    return cudaSuccess;
 }
 
 cudaError_t launch_route_bwd(const RouteBwdArgs& a, bool bf16, void* ws, cudaStream_t s) {
-    return bf16 ? launch_route_bwd_t<__nv_bfloat16>(a, ws, s) : launch_route_bwd_t<float>(a, ws, s);
+    return bf16 ? launch_route_bwd_tc(a, ws, s) : launch_route_bwd_simt(a, ws, s);
 }
 
 cudaError_t route_status(cudaStream_t s, int* code) { return tu_status_read_clear(s, code); }

@@ -65,6 +65,7 @@ class MoELayer:
         self.dlogits = z(T, E, dtype=f32)
         self.dw_router = z(P, E, d)
         self.dbias = z(P, E, dtype=f32)
+        self.dx_router = z(T, d)
         self.dx = z(T, d)
         # the aux loss and the router backward run beside the expert GEMMs on this stream
         self.side = torch.cuda.Stream(device=device)
@@ -135,8 +136,8 @@ class MoELayer:
         self.side.wait_event(fork)
         L.moe_route_bwd(c, self.x, self.w_router, self.probs, self.topk_idx, self.topk_w,
                         self.dtopk_w, self.aux_coef if with_aux else None, self._po(),
-                        self.dlogits, self.dw_router, self.dbias, self.workspace, self.ws_bytes,
-                        stream=self.side)
+                        self.dlogits, self.dw_router, self.dbias, self.dx_router, self.workspace,
+                        self.ws_bytes, stream=self.side)
         join = torch.cuda.Event()
         join.record(self.side)
         mark("ffn_bwd_begin")
@@ -146,8 +147,8 @@ class MoELayer:
                              self.dx_sh, self.dws1, self.dws2, stream=main)
         mark("ffn_bwd_end")
         main.wait_event(join)
-        L.moe_dispatch_bwd(c, self.dx_perm, self.slot_of, self.dlogits, self.w_router, self._po(),
-                           self.dx_sh, self.dx, stream=main)
+        L.moe_dispatch_bwd(c, self.dx_perm, self.slot_of, self.dx_router, self.dx_sh, self.dx,
+                           stream=main)
 
     def step(self, stream=None, mark=None):
         """One fwd+bwd pass of the whole layer. ``mark(name)`` (optional) is called at
@@ -191,8 +192,11 @@ class MoELayer:
     def kernels_per_step(self) -> int:
         """CUDA kernels this library launches per step (memsets not counted):
         route 1, aux 1, dispatch 3, expert fwd 2, combine 1, combine bwd 1,
-        expert bwd 4, route bwd 2, unpermute-reduce 1; shared experts add 2 + 4."""
-        return 16 + (6 if self.shape.n_shared else 0)
+        expert bwd 4, unpermute-reduce 1, and the router backward: bf16 5 (dlogits,
+        chunk dbias, dW_r partial GEMM, reduce, dx_router GEMM), fp32 4 (dlogits,
+        partials, reduce, dx_router GEMM); shared experts add 2 + 4."""
+        rb = 5 if self.shape.dtype == "bf16" else 4
+        return 14 + rb + (6 if self.shape.n_shared else 0)
 
     def check_status(self, stream=None):
         code = L.moe_device_status(stream)

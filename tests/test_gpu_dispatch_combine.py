@@ -113,27 +113,25 @@ def test_combine_fwd_bwd(L, T, E, k, S, dtype):
 @pytest.mark.parametrize("T,E,k,P,S,dtype", [(700, 8, 2, 1, 0, "bf16"), (400, 32, 2, 4, 0, "bf16"),
                                              (300, 64, 6, 1, 2, "bf16"), (256, 8, 2, 2, 1, "f32")])
 def test_unpermute_reduce_with_router_grad(L, T, E, k, P, S, dtype):
+    """dx = the k permuted rows of each token + the router's share + the shared experts'."""
     d = 512
     idx, counts, off, slot, tok = _tables(T, E, k, 5)
     rng = np.random.default_rng(6)
     rnd = (lambda *s: mi.bf16_round(rng.standard_normal(s).astype(np.float32))) if dtype == "bf16" \
         else (lambda *s: rng.standard_normal(s).astype(np.float32))
-    dxp, dxsh = rnd(T * k, d), rnd(S, T, d)
-    wr = rnd(P, E, d) * np.float32(0.02) if dtype == "f32" else mi.bf16_round(rnd(P, E, d) * np.float32(0.02))
-    dz = rng.standard_normal((T, E)).astype(np.float32)
-    po = np.linspace(0, T, P + 1).astype(np.int32)
+    dxp, dxsh, dxr = rnd(T * k, d), rnd(S, T, d), rnd(T, d)
     sh = mi.MoEShape("u", T, d, E, 256, k, dtype, n_parties=P, n_shared=S, d_ff_shared=128 if S else 0)
     cfg = cfg_of(L, sh)
     dt = torch.bfloat16 if dtype == "bf16" else torch.float32
-    dx = empty((T, d), dt)
-    L.moe_dispatch_bwd(cfg, dev(dxp, dt), dev(slot.ravel(), torch.int32), dev(dz, torch.float32),
-                       dev(wr, dt), dev(po, torch.int32) if P > 1 else None,
-                       dev(dxsh, dt) if S else None, dx)
-    assert status(L) == 0
-    ref = mo.unpermute_reduce(dxp.astype(np.float64), slot) + dxsh.astype(np.float64).sum(0)
-    part = mo.party_of_tokens(T, po)
-    ref += np.einsum("te,ted->td", dz.astype(np.float64), wr.astype(np.float64)[part])
-    assert_close("dx", dx, ref, 1e-5 if dtype == "f32" else 8e-3)
+    for with_router in (True, False):
+        dx = empty((T, d), dt)
+        L.moe_dispatch_bwd(cfg, dev(dxp, dt), dev(slot.ravel(), torch.int32),
+                           dev(dxr, dt) if with_router else None, dev(dxsh, dt) if S else None, dx)
+        assert status(L) == 0
+        ref = mo.unpermute_reduce(dxp.astype(np.float64), slot) + dxsh.astype(np.float64).sum(0)
+        if with_router:
+            ref += dxr.astype(np.float64)
+        assert_close("dx", dx, ref, 1e-5 if dtype == "f32" else 8e-3)
 
 
 def test_combine_detects_bad_slot(L):

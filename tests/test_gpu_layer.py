@@ -55,7 +55,8 @@ def full_compare(lay, inp, sh):
         ("dh", lay.dh, bwd["dh"]), ("dx_perm", lay.dx_perm, bwd["dx_perm"]),
         ("dw1", lay.dw1, bwd["dw1"]), ("dw2", lay.dw2, bwd["dw2"]),
         ("dlogits", lay.dlogits, bwd["dlogits"]), ("dw_router", lay.dw_router, bwd["dw_router"]),
-        ("dbias", lay.dbias, bwd["dbias"]), ("dx", lay.dx, bwd["dx"]),
+        ("dbias", lay.dbias, bwd["dbias"]), ("dx_router", lay.dx_router, bwd["dx_router"]),
+        ("dx", lay.dx, bwd["dx"]),
     ]:
         errs[name] = assert_close(name, gpu, ref, tol)
     for s in range(sh.n_shared):
@@ -174,6 +175,10 @@ def test_layer_sampled_parity_full_size(L, which):
     assert_close("dx", lay.dx[toks_d], rows["dx"], tol)
     assert_close("dtopk_w", lay.dtopk_w[toks_d], rows["dtopk_w"], tol)
     assert_close("dlogits", lay.dlogits[toks_d], rows["dlogits"], tol)
+    part = mo.party_of_tokens(sh.T, inp["party_offsets"])[toks]
+    wr = np.asarray(inp["w_router"], np.float64)
+    ref_dxr = np.einsum("te,ted->td", np.asarray(rows["dlogits"], np.float64), wr[part])
+    assert_close("dx_router", lay.dx_router[toks_d], ref_dxr, tol)
     slot = ints(lay.slot_of).reshape(sh.T, sh.top_k)
     for i, t in enumerate(toks):
         assert_close("y", lay.y_perm[torch.as_tensor(slot[t], device="cuda")], rows["y"][i], tol)
