@@ -315,6 +315,7 @@ struct Tile {
     int64_t out_row;    // M-var: output row of group row 0
     int k_iters;
     int last_rows;      // K-var: valid contraction rows in the last k-block (1..64)
+    bool dw;            // a tile of the second (K-variable) problem of a fused launch
 };
 
 // ------------------------------------------------------------------------ router epilogue
@@ -397,13 +398,23 @@ __device__ __forceinline__ void route_epilogue(const Params& p, const Tile& ti, 
 // PAIR: the two CTAs of a cluster compute one 256 x BN tile with tcgen05 cta_group::2
 // MMAs issued by CTA 0: each CTA holds 128 rows of A and BN/2 rows of B in its own
 // shared memory and 128 rows of the accumulator in its own TMEM.
-template <int BN, bool B_MN, bool VAR_K, int EPI, bool PAIR = false>
+// DW2: the launch also computes a second, K-variable problem with the same groups
+// (p2, tmA2, tmB2, tmO2: C_g = A_g^T B_g over group g's rows, MN-major operands, bf16
+// store), its tiles after all of the first problem's: one persistent launch, one tail,
+// for a weight gradient and the M-variable GEMM of the same backward step. (Interleaving
+// the two problems' tiles group by group measured slower: a tile with a long epilogue
+// followed by one with a short mainloop leaves the MMA waiting for an accumulator.)
+template <int BN, bool B_MN, bool VAR_K, int EPI, bool PAIR = false, bool DW2 = false>
 __global__ void __launch_bounds__(THREADS, 1)
     grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA,
                         const __grid_constant__ CUtensorMap tmB,
                         const __grid_constant__ CUtensorMap tmO0,
-                        const __grid_constant__ CUtensorMap tmO1, const Params p) {
+                        const __grid_constant__ CUtensorMap tmO1, const Params p,
+                        const __grid_constant__ CUtensorMap tmA2,
+                        const __grid_constant__ CUtensorMap tmB2,
+                        const __grid_constant__ CUtensorMap tmO2, const Params p2) {
     pdl_begin();
+    static_assert(!DW2 || (B_MN && !VAR_K && !PAIR && BN == 256), "fused: M-variable, MN-major B");
     constexpr bool A_MN = VAR_K;
     constexpr int NPAIR = PAIR ? 2 : 1;
     constexpr int BNL = BN / NPAIR;  // B rows held by this CTA
@@ -413,6 +424,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
     constexpr int NST = num_stages(STAGE_BYTES, EPI);
     constexpr uint32_t IDESC = instr_desc<BN, A_MN, B_MN, BMP>();
+    constexpr uint32_t IDESC_DW = instr_desc<BN, true, true, BM>();
     constexpr int TMEM_COLS = (2 * BN <= 32) ? 32 : (2 * BN <= 64) ? 64 : (2 * BN <= 128) ? 128 : (2 * BN <= 256) ? 256 : 512;
 
     extern __shared__ uint8_t smem_raw[];
@@ -420,6 +432,9 @@ __global__ void __launch_bounds__(THREADS, 1)
     __shared__ uint32_t s_tmem;
     __shared__ int s_abort;
     __shared__ int s_tile_start[MAX_GROUPS + 1];
+    __shared__ int s_total1;  // fused: tiles of the first problem
+    __shared__ unsigned char s_order[DW2 ? MAX_GROUPS : 1];  // fused: second problem's group order
+    __shared__ int s_rows[DW2 ? MAX_GROUPS : 1];
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     volatile int* abort_flag = &s_abort;
@@ -442,14 +457,50 @@ __global__ void __launch_bounds__(THREADS, 1)
             acc += mt * tiles_n;
         }
         s_tile_start[p.G] = acc;
+        s_total1 = acc;
+        if constexpr (DW2) s_tile_start[p.G] = acc + p.G * (p2.Mout / BM) * (p2.N / BN);
         s_abort = 0;
     }
+    if constexpr (DW2) {
+        for (int g = threadIdx.x; g < p2.G; g += blockDim.x) s_rows[g] = p2.offsets[g + 1] - p2.offsets[g];
+    }
     __syncthreads();
+    if constexpr (DW2) {
+        // weight-gradient groups longest first (each tile of a group runs over all its
+        // rows): with skewed experts the long tiles then do not form the tail. Rank of g =
+        // groups with more rows, or as many and a lower index.
+        for (int g = threadIdx.x; g < p2.G; g += blockDim.x) {
+            int rank = 0;
+            for (int h = 0; h < p2.G; ++h)
+                rank += (s_rows[h] > s_rows[g]) || (s_rows[h] == s_rows[g] && h < g);
+            s_order[rank] = (unsigned char)g;
+        }
+        __syncthreads();
+    }
     const int total_tiles = s_tile_start[p.G];
     if (tile0 >= total_tiles) return;  // uniform across the pair
 
     auto tile_at = [&](int t) -> Tile {
         Tile ti;
+        ti.dw = false;
+        if constexpr (DW2) {
+            if (t >= s_total1) {  // second problem: K-variable, rows of group g
+                const int per = (p2.Mout / BM) * (p2.N / BN);
+                const int g = s_order[(t - s_total1) / per], l2 = (t - s_total1) % per;
+                const int tn2 = p2.N / BN;
+                ti.dw = true;
+                ti.g = g;
+                ti.m0 = (l2 / tn2) * BM;
+                ti.n0 = (l2 % tn2) * BN;
+                const int64_t r0 = p2.offsets[g], nrows = p2.offsets[g + 1] - r0;
+                ti.mvalid = p2.Mout;
+                ti.a_row = ti.b_row = r0;
+                ti.out_row = 0;
+                ti.k_iters = (int)((nrows + BK - 1) / BK);
+                ti.last_rows = (int)(nrows - (int64_t)(ti.k_iters - 1) * BK);
+                return ti;
+            }
+        }
         int g = 0;
         while (g + 1 < p.G && s_tile_start[g + 1] <= t) ++g;
         const int local = t - s_tile_start[g];
@@ -592,12 +643,14 @@ __global__ void __launch_bounds__(THREADS, 1)
                         mbar_expect_tx(fb, STAGE_BYTES);
                     }
                     const int k0 = kb * BK;
-                    if (!A_MN) {
+                    const bool dw = DW2 && ti.dw;
+                    if (!A_MN && !dw) {
                         load(sa, &tmA, fb, k0, (int)(ti.a_row + ti.m0));
                     } else {
+                        const CUtensorMap* mA = dw ? &tmA2 : &tmA;
 #pragma unroll
                         for (int i = 0; i < BM / 64; ++i)
-                            load(sa + i * 8192, &tmA, fb, ti.m0 + 64 * i, (int)(ti.a_row + k0));
+                            load(sa + i * 8192, mA, fb, ti.m0 + 64 * i, (int)(ti.a_row + k0));
                     }
                     if (EPI == EPI_SWIGLU_FWD) {
                         // 128 gate rows then 128 up rows of the same features; in a pair the
@@ -612,10 +665,11 @@ __global__ void __launch_bounds__(THREADS, 1)
                     } else if (!B_MN) {
                         load(sb, &tmB, fb, k0, (int)((int64_t)ti.g * p.b_group_rows + ti.n0 + rank * BNL));
                     } else {
-                        const int64_t krow = VAR_K ? (ti.b_row + k0) : ((int64_t)ti.g * p.b_group_rows + k0);
+                        const int64_t krow = (VAR_K || dw) ? (ti.b_row + k0) : ((int64_t)ti.g * p.b_group_rows + k0);
+                        const CUtensorMap* mB = dw ? &tmB2 : &tmB;
 #pragma unroll
                         for (int i = 0; i < BNL / 64; ++i)
-                            load(sb + i * 8192, &tmB, fb, ti.n0 + (int)rank * BNL + 64 * i, (int)krow);
+                            load(sb + i * 8192, mB, fb, ti.n0 + (int)rank * BNL + 64 * i, (int)krow);
                     }
                     issued_phase[stage] = (int)phase;
                     if (++stage == NST) {
@@ -666,7 +720,8 @@ __global__ void __launch_bounds__(THREADS, 1)
                 // last of them the A rows past the group's end are zeroed (A alone suffices:
                 // their products with any finite B row vanish).
                 int ksteps = BK / 16;
-                if (VAR_K && kb == ti.k_iters - 1 && ti.last_rows < BK) {
+                const bool dwt = DW2 && ti.dw;
+                if ((VAR_K || dwt) && kb == ti.k_iters - 1 && ti.last_rows < BK) {
                     ksteps = (ti.last_rows + 15) / 16;
                     const int zr0 = ti.last_rows, zr1 = ksteps * 16;
                     if (zr1 > zr0) {
@@ -687,12 +742,12 @@ __global__ void __launch_bounds__(THREADS, 1)
                     for (int kk = 0; kk < BK / 16; ++kk) {
                         if (kk >= ksteps) break;
                         uint64_t ad, bd;
-                        if (!A_MN) ad = smem_desc(sa + kk * 32, 16, 1024);
+                        if (!A_MN && !dwt) ad = smem_desc(sa + kk * 32, 16, 1024);
                         else ad = smem_desc(sa + kk * 2048, 8192, 1024);
                         if (!B_MN) bd = smem_desc(sb + kk * 32, 16, 1024);
                         else bd = smem_desc(sb + kk * 2048, 8192, 1024);
                         if constexpr (PAIR) mma_bf16_pair(tmem_d, ad, bd, IDESC, (kb | kk) ? 1u : 0u);
-                        else mma_bf16(tmem_d, ad, bd, IDESC, (kb | kk) ? 1u : 0u);
+                        else mma_bf16(tmem_d, ad, bd, dwt ? IDESC_DW : IDESC, (kb | kk) ? 1u : 0u);
                     }
                     if constexpr (PAIR) mma_commit_pair(empty_bar(stage), 3);  // both producers
                     else mma_commit(empty_bar(stage));
@@ -762,7 +817,10 @@ __global__ void __launch_bounds__(THREADS, 1)
             return mbar_wait(gu_bar0 + 8u * b, parity, abort_flag, limit);
         };
         if constexpr (EPI == EPI_SWIGLU_BWD) {
-            if (tile0 < total_tiles) gu_issue(tile_at(tile0), 0);
+            if (tile0 < total_tiles) {
+                const Tile tf = tile_at(tile0);
+                if (!(DW2 && tf.dw)) gu_issue(tf, 0);
+            }
         }
         for (int t = tile0; t < total_tiles; t += tile_step) {
             const Tile ti = tile_at(t);
@@ -770,7 +828,9 @@ __global__ void __launch_bounds__(THREADS, 1)
             const bool valid = m < ti.mvalid;
             const int wrow0 = ti.m0 + q * 32;
             const bool full_box = wrow0 + 32 <= ti.mvalid;
-            const int64_t grow0 = VAR_K ? (int64_t)ti.g * p.Mout + wrow0 : ti.out_row + wrow0;
+            const bool dwt = DW2 && ti.dw;
+            const int64_t grow0 = (VAR_K || dwt) ? (int64_t)ti.g * (dwt ? p2.Mout : p.Mout) + wrow0
+                                                 : ti.out_row + wrow0;
             const uint32_t tbase = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
             // write NOUT rows of 32 values each: staged + TMA when the whole box is valid
             auto emit = [&](int nout, const float* const* vals, const CUtensorMap* const* maps,
@@ -795,13 +855,34 @@ __global__ void __launch_bounds__(THREADS, 1)
                     for (int o = 0; o < nout; ++o) store_row32(direct[o], vals[o]);
                 }
             };
-            if constexpr (EPI == EPI_SWIGLU_BWD) {
+            if (dwt) {
+                // second problem: a bf16 weight-gradient tile, [Mout, N] per group
+                if (!wait_bar(tfull_bar(acc), acc_phase)) break;
+                fence_after();
+                __nv_bfloat16* out = (__nv_bfloat16*)p2.out0 + (int64_t)ti.g * p2.Mout * p2.N + (int64_t)m * p2.N;
+#pragma unroll 1
+                for (int c = 0; c < BN; c += 32) {
+                    float y[32];
+                    if (ti.k_iters > 0) {
+                        tmem_ld32(tbase + c, y);
+                    } else {
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) y[i] = 0.f;
+                    }
+                    const float* vals[1] = {y};
+                    const CUtensorMap* maps[1] = {&tmO2};
+                    const int cols[1] = {ti.n0 + c};
+                    __nv_bfloat16* direct[1] = {out + ti.n0 + c};
+                    emit(1, vals, maps, cols, direct);
+                }
+            } else if constexpr (EPI == EPI_SWIGLU_BWD) {
                 // dA in TMEM. G and U of each 32-column chunk arrive by TMA in one of two
                 // staging buffers (the next chunk's load is in flight while this one is
                 // computed); dG and dU overwrite them in place and leave by TMA store.
                 const int F = p.F;
                 __nv_bfloat16* dh = (__nv_bfloat16*)p.out0 + (ti.out_row + m) * (int64_t)(2 * F) + ti.n0;
                 constexpr int NCH = BN / 32;
+                if (gu_issued == gu_chunk) gu_issue(ti, 0);  // not prefetched (a fused tile came before)
                 if (!wait_bar(tfull_bar(acc), acc_phase)) break;
                 fence_after();
                 bool stop = false;
@@ -809,7 +890,10 @@ __global__ void __launch_bounds__(THREADS, 1)
                 for (int c = 0; c < NCH; ++c) {
                     // prefetch the next chunk (of this tile, or the first of the next tile)
                     if (c + 1 < NCH) gu_issue(ti, c + 1);
-                    else if (t + tile_step < total_tiles) gu_issue(tile_at(t + tile_step), 0);
+                    else if (t + tile_step < total_tiles) {
+                        const Tile tn = tile_at(t + tile_step);
+                        if (!(DW2 && tn.dw)) gu_issue(tn, 0);
+                    }
                     const int b = gu_chunk & 1;
                     if (!gu_wait(b, (gu_chunk >> 1) & 1)) { stop = true; break; }
                     uint8_t* gbuf = stg + (2 * b) * EPI_BUF_BYTES + lane * 64;
@@ -1008,11 +1092,17 @@ static int sm_count() {
     return n;
 }
 
-template <int BN, bool B_MN, bool VAR_K, int EPI, bool PAIR = false>
+template <int BN, bool B_MN, bool VAR_K, int EPI, bool PAIR = false, bool DW2 = false>
 static cudaError_t launch(const CUtensorMap& ma, const CUtensorMap& mb, const CUtensorMap& mo0,
                           const CUtensorMap& mo1, const Params& p, int64_t tiles_ub,
-                          cudaStream_t s) {
-    auto kern = grouped_gemm_kernel<BN, B_MN, VAR_K, EPI, PAIR>;
+                          cudaStream_t s, const CUtensorMap* ma2 = nullptr,
+                          const CUtensorMap* mb2 = nullptr, const CUtensorMap* mo2 = nullptr,
+                          const Params* p2 = nullptr) {
+    auto kern = grouped_gemm_kernel<BN, B_MN, VAR_K, EPI, PAIR, DW2>;
+    const CUtensorMap& A2 = ma2 ? *ma2 : ma;
+    const CUtensorMap& B2 = mb2 ? *mb2 : mb;
+    const CUtensorMap& O2 = mo2 ? *mo2 : mo0;
+    const Params& P2 = p2 ? *p2 : p;
     constexpr int NPAIR = PAIR ? 2 : 1;
     constexpr int NST = num_stages((uint32_t)(BM * BK * 2 + BN / NPAIR * BK * 2), EPI);
     const int extra_max = EPI == EPI_ROUTE ? 64 * 64 * 4 : EPI_WARPS * epi_stage_bytes(EPI);
@@ -1064,10 +1154,10 @@ static cudaError_t launch(const CUtensorMap& ma, const CUtensorMap& mb, const CU
         attr[1].val.programmaticStreamSerializationAllowed = 1;
         cfg.attrs = attr;
         cfg.numAttrs = 2;
-        return cudaLaunchKernelEx(&cfg, kern, ma, mb, mo0, mo1, p);
+        return cudaLaunchKernelEx(&cfg, kern, ma, mb, mo0, mo1, p, A2, B2, O2, P2);
     } else {
         const int grid = (int)std::min<int64_t>(tiles_ub, sm_count());
-        (void)launch_pdl(kern, dim3(grid), dim3(THREADS), smem, s, ma, mb, mo0, mo1, p);
+        (void)launch_pdl(kern, dim3(grid), dim3(THREADS), smem, s, ma, mb, mo0, mo1, p, A2, B2, O2, P2);
         return cudaGetLastError();
     }
 }
@@ -1076,6 +1166,18 @@ static cudaError_t launch(const CUtensorMap& ma, const CUtensorMap& mb, const CU
 
 void set_wait_limit_ns(uint64_t ns) { tc::g_wait_ns = ns ? ns : 1; }
 void set_gemm_pairs(int mode) { tc::g_pairs = mode; }
+
+// Pair tiles where they fill at least four rounds of the SMs (the last, partly empty
+// round then costs little) and the operand feed, not the epilogue, bounds the tile.
+bool gemm_m_uses_pairs(const GemmMArgs& g) {
+    using namespace tc;
+    if (g.N % 256 != 0) return false;
+    if (g_pairs == MOE_PAIRS_ALL) return true;
+    if (g_pairs != MOE_PAIRS_AUTO || g.epi == EPI_SWIGLU_BWD) return false;
+    const int64_t pt_ub = g.rows.offsets ? ((int64_t)g.rows.rows + 2 * BM - 1) / (2 * BM) + g.G
+                                         : (int64_t)g.G * ((g.rows.rows + 2 * BM - 1) / (2 * BM));
+    return pt_ub * (g.N / 256) >= 4 * (int64_t)(sm_count() / 2);
+}
 
 // M-variable grouped GEMM (forward, dA, dX).
 cudaError_t launch_gemm_m(const GemmMArgs& g, bool bf16, cudaStream_t s) {
@@ -1103,13 +1205,7 @@ cudaError_t launch_gemm_m(const GemmMArgs& g, bool bf16, cudaStream_t s) {
     // pair tiles (256 rows)
     const int64_t pt_ub = g.rows.offsets ? ((int64_t)g.rows.rows + 2 * BM - 1) / (2 * BM) + g.G
                                          : (int64_t)g.G * ((g.rows.rows + 2 * BM - 1) / (2 * BM));
-    // pair tiles where they fill at least four rounds of the SMs (the last, partly empty
-    // round then costs little) and the operand feed, not the epilogue, bounds the tile
-    const int64_t pair_tiles = pt_ub * (g.N / 256);
-    const bool pair = g.N % 256 == 0 &&
-                      (g_pairs == MOE_PAIRS_ALL ||
-                       (g_pairs == MOE_PAIRS_AUTO && g.epi != EPI_SWIGLU_BWD &&
-                        pair_tiles >= 4 * (int64_t)(sm_count() / 2)));
+    const bool pair = gemm_m_uses_pairs(g);
     // output rows in the 2D view of the outputs
     const int64_t o_rows = g.rows.offsets ? (int64_t)g.rows.rows
                                           : std::max<int64_t>(g.rows.rows, (int64_t)(g.G - 1) * g.rows.out_stride + g.rows.rows);
@@ -1191,6 +1287,64 @@ cudaError_t launch_gemm_k(const GemmKArgs& g, bool bf16, cudaStream_t s) {
     if (!make_map(&mo, g.out, g.N, (int64_t)g.G * g.M, 0, true)) return cudaErrorInvalidValue;
     if (g.N % 256 == 0) return launch<256, true, true, EPI_STORE>(ma, mb, mo, mo, p, tiles * (g.N / 256), s);
     return launch<128, true, true, EPI_STORE>(ma, mb, mo, mo, p, tiles * (g.N / 128), s);
+}
+
+// One launch of an M-variable GEMM with MN-major B (dA with the SwiGLU-backward
+// epilogue, or dX) and a K-variable weight-gradient GEMM over the same groups (dW2, or
+// dW1); see the DW2 kernel parameter. Falls back to two
+// launches when the shapes do not fit one 256-wide template.
+cudaError_t launch_gemm_mk(const GemmMArgs& g, const GemmKArgs& k, cudaStream_t s) {
+    using namespace tc;
+    const bool fits = g.rows.offsets && k.rows.offsets && g.G == k.G && !g.b_kmajor &&
+                      (g.epi == EPI_SWIGLU_BWD || g.epi == EPI_STORE) && g.N % 256 == 0 &&
+                      k.N % 256 == 0 && k.M % BM == 0 && k.epi == EPI_STORE && g.G <= MAX_GROUPS;
+    if (!fits) {
+        cudaError_t e = launch_gemm_m(g, true, s);
+        if (e != cudaSuccess) return e;
+        return launch_gemm_k(k, true, s);
+    }
+    // first problem (as launch_gemm_m, MN-major B)
+    Params p{};
+    p.offsets = g.rows.offsets;
+    p.G = g.G;
+    p.N = g.N;
+    p.K = g.K;
+    p.out0 = g.out0;
+    p.out1 = g.out1;
+    p.aux = g.aux;
+    p.wait_ns = g_wait_ns;
+    p.b_group_rows = g.b_rows ? g.b_rows : g.K;
+    const int64_t a_rows = (int64_t)g.rows.rows, o_rows = a_rows;
+    CUtensorMap ma, mb, mo0, mo1;
+    if (!make_map(&ma, g.a, g.K, a_rows, BM)) return cudaErrorInvalidValue;
+    if (!make_map(&mb, g.b, g.N, (int64_t)g.G * p.b_group_rows, 64)) return cudaErrorInvalidValue;
+    if (g.epi == EPI_SWIGLU_BWD) {
+        p.F = g.N;
+        if (!make_map(&mo0, g.out0, 2 * (int64_t)g.N, o_rows, 0, true)) return cudaErrorInvalidValue;
+        if (!make_map(&mo1, g.aux, 2 * (int64_t)g.N, o_rows, 0, true)) return cudaErrorInvalidValue;
+    } else {
+        if (!make_map(&mo0, g.out0, g.N, o_rows, 0, true)) return cudaErrorInvalidValue;
+        mo1 = mo0;
+    }
+    // second problem (as launch_gemm_k)
+    Params p2{};
+    p2.offsets = k.rows.offsets;
+    p2.G = k.G;
+    p2.N = k.N;
+    p2.Mout = k.M;
+    p2.out0 = k.out;
+    p2.wait_ns = g_wait_ns;
+    CUtensorMap ma2, mb2, mo2;
+    if (!make_map(&ma2, k.a, k.M, (int64_t)k.rows.rows, 64)) return cudaErrorInvalidValue;
+    if (!make_map(&mb2, k.b, k.N, (int64_t)k.rows.rows, 64)) return cudaErrorInvalidValue;
+    if (!make_map(&mo2, k.out, k.N, (int64_t)k.G * k.M, 0, true)) return cudaErrorInvalidValue;
+    const int64_t tiles = (((int64_t)g.rows.rows + BM - 1) / BM + g.G) * (g.N / 256) +
+                          (int64_t)k.G * (k.M / BM) * (k.N / 256);
+    if (g.epi == EPI_SWIGLU_BWD)
+        return launch<256, true, false, EPI_SWIGLU_BWD, false, true>(ma, mb, mo0, mo1, p, tiles, s,
+                                                                     &ma2, &mb2, &mo2, &p2);
+    return launch<256, true, false, EPI_STORE, false, true>(ma, mb, mo0, mo1, p, tiles, s, &ma2,
+                                                            &mb2, &mo2, &p2);
 }
 
 // Router logits on the tensor cores with the gating epilogue: groups are parties

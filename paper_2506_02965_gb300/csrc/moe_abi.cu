@@ -491,20 +491,37 @@ moe_status moe_expert_ffn_bwd(const moe_config* cfg, const void* x_perm, const i
     w1g.M = 2 * F;
     w1g.N = d;
     w1g.out = dw1;
-    // caller stream: dA then dX; side stream: dW2 (needs only dY and A) alongside dA,
-    // then dW1 once dH exists
+    // Each M-variable GEMM runs with its weight gradient in one persistent launch (one
+    // tail instead of two, and no two persistent grids contending for SMs): dA then dW2
+    // (which needs only dY and A), dX then dW1 (which needs dH). A GEMM that runs as
+    // CTA-pair tiles, and the CUDA-core path, instead put the weight gradient on a side
+    // stream: dW2 alongside dA, dW1 alongside dX once dH exists.
+    const bool fuse_a = bf16 && !gemm_m_uses_pairs(a);
+    const bool fuse_b = bf16 && !gemm_m_uses_pairs(b);
     SideStream* ss = nullptr;
-    if ((st = cuda_status(side_stream(&ss), "side stream"))) return st;
-    if ((st = cuda_status(cudaEventRecord(ss->fork, s), "fork"))) return st;
-    if ((st = cuda_status(cudaStreamWaitEvent(ss->s, ss->fork, 0), "fork"))) return st;
-    if ((st = cuda_status(launch_gemm_k(w2g, bf16, ss->s), "expert dW2 gemm"))) return st;
-    if ((st = cuda_status(launch_gemm_m(a, bf16, s), "expert dA gemm"))) return st;
-    if ((st = cuda_status(cudaEventRecord(ss->mid, s), "mid"))) return st;
-    if ((st = cuda_status(launch_gemm_m(b, bf16, s), "expert dX gemm"))) return st;
-    if ((st = cuda_status(cudaStreamWaitEvent(ss->s, ss->mid, 0), "mid"))) return st;
-    if ((st = cuda_status(launch_gemm_k(w1g, bf16, ss->s), "expert dW1 gemm"))) return st;
-    if ((st = cuda_status(cudaEventRecord(ss->join, ss->s), "join"))) return st;
-    if ((st = cuda_status(cudaStreamWaitEvent(s, ss->join, 0), "join"))) return st;
+    if (!fuse_a || !fuse_b) {
+        if ((st = cuda_status(side_stream(&ss), "side stream"))) return st;
+        if ((st = cuda_status(cudaEventRecord(ss->fork, s), "fork"))) return st;
+        if ((st = cuda_status(cudaStreamWaitEvent(ss->s, ss->fork, 0), "fork"))) return st;
+    }
+    if (fuse_a) {
+        if ((st = cuda_status(launch_gemm_mk(a, w2g, s), "expert dA+dW2 gemm"))) return st;
+    } else {
+        if ((st = cuda_status(launch_gemm_k(w2g, bf16, ss->s), "expert dW2 gemm"))) return st;
+        if ((st = cuda_status(launch_gemm_m(a, bf16, s), "expert dA gemm"))) return st;
+    }
+    if (fuse_b) {
+        if ((st = cuda_status(launch_gemm_mk(b, w1g, s), "expert dX+dW1 gemm"))) return st;
+    } else {
+        if ((st = cuda_status(cudaEventRecord(ss->mid, s), "mid"))) return st;
+        if ((st = cuda_status(launch_gemm_m(b, bf16, s), "expert dX gemm"))) return st;
+        if ((st = cuda_status(cudaStreamWaitEvent(ss->s, ss->mid, 0), "mid"))) return st;
+        if ((st = cuda_status(launch_gemm_k(w1g, bf16, ss->s), "expert dW1 gemm"))) return st;
+    }
+    if (ss) {
+        if ((st = cuda_status(cudaEventRecord(ss->join, ss->s), "join"))) return st;
+        if ((st = cuda_status(cudaStreamWaitEvent(s, ss->join, 0), "join"))) return st;
+    }
     if (S) {
         GemmMArgs sa = a;
         sa.G = S;

@@ -129,6 +129,11 @@ struct GemmKArgs {
 
 cudaError_t launch_gemm_m(const GemmMArgs& g, bool bf16, cudaStream_t s);
 cudaError_t launch_gemm_k(const GemmKArgs& g, bool bf16, cudaStream_t s);
+// bf16: an M-variable GEMM (MN-major B) and a K-variable GEMM over the same groups in
+// one persistent launch (the second problem's tiles after the first's)
+cudaError_t launch_gemm_mk(const GemmMArgs& m, const GemmKArgs& k, cudaStream_t s);
+// whether launch_gemm_m runs this GEMM as CTA-pair tiles (bf16)
+bool gemm_m_uses_pairs(const GemmMArgs& g);
 void set_wait_limit_ns(uint64_t ns);
 void set_gemm_pairs(int mode);  // MOE_PAIRS_*
 cudaError_t gemm_status(cudaStream_t s, int* code);
