@@ -306,8 +306,9 @@ __global__ void __launch_bounds__(256) dlogits_kernel(
     }
 }
 
-// dbias partial of one token chunk: part_db[c][e] = sum of dlogits[t][e] over the chunk,
-// four token strides summed in a fixed order.
+// dbias partial of one token chunk: part_db[c][e] = sum of dlogits[t][e] over the chunk.
+// Thread group g (of 4) takes tokens g, g+4, ... with eight independent accumulators
+// (eight loads in flight), summed in a fixed order, then the four groups in order.
 __global__ void __launch_bounds__(256) chunk_db_kernel(const float* __restrict__ dz,
                                                       const int32_t* __restrict__ chunk_off, int E,
                                                       float* part_db) {
@@ -316,8 +317,16 @@ __global__ void __launch_bounds__(256) chunk_db_kernel(const float* __restrict__
     const int c = blockIdx.x, e = threadIdx.x & 63, g = threadIdx.x >> 6;
     const int64_t a = chunk_off[c], b = chunk_off[c + 1];
     float acc = 0.f;
-    if (e < E)
-        for (int64_t t = a + g; t < b; t += 4) acc += dz[t * E + e];
+    if (e < E) {
+        float u[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+        int64_t t = a + g;
+        for (; t + 28 < b; t += 32) {
+#pragma unroll
+            for (int i = 0; i < 8; ++i) u[i] += dz[(t + 4 * i) * E + e];
+        }
+        for (; t < b; t += 4) u[0] += dz[t * E + e];
+        acc = ((u[0] + u[1]) + (u[2] + u[3])) + ((u[4] + u[5]) + (u[6] + u[7]));
+    }
     s_part[g][e] = acc;
     __syncthreads();
     if (g == 0 && e < E) part_db[(int64_t)c * E + e] = ((s_part[0][e] + s_part[1][e]) + s_part[2][e]) + s_part[3][e];
@@ -523,7 +532,8 @@ struct RbTcLayout {
     size_t dw, db, off, dz, total;
 };
 // Tokens per chunk of the chunked dW_r contraction: about 256 tiles of 128 model columns
-// in all, at most 128 - P chunks (the grouped GEMM's group limit), a multiple of 64.
+// in all (one wave of 152 measured slower), at most 128 - P chunks (the grouped GEMM's
+// group limit), a multiple of 64.
 static RbTcLayout rb_tc_layout(int64_t T, int P, int E, int d) {
     RbTcLayout L;
     const int64_t mt = std::max(1, d / 128);
