@@ -307,29 +307,25 @@ __global__ void __launch_bounds__(256) dlogits_kernel(
 }
 
 // dbias partial of one token chunk: part_db[c][e] = sum of dlogits[t][e] over the chunk.
-// Thread group g (of 4) takes tokens g, g+4, ... with eight independent accumulators
-// (eight loads in flight), summed in a fixed order, then the four groups in order.
+// Thread (g, e) of a block, g < G = 256 / E token groups, sums tokens g, g + G, ...; the
+// groups are then added in order (fixed order: deterministic).
 __global__ void __launch_bounds__(256) chunk_db_kernel(const float* __restrict__ dz,
                                                       const int32_t* __restrict__ chunk_off, int E,
                                                       float* part_db) {
     pdl_begin();
-    __shared__ float s_part[4][64];
-    const int c = blockIdx.x, e = threadIdx.x & 63, g = threadIdx.x >> 6;
+    __shared__ float s_part[256];
+    const int c = blockIdx.x, G = 256 / E, e = threadIdx.x % E, g = threadIdx.x / E;
     const int64_t a = chunk_off[c], b = chunk_off[c + 1];
     float acc = 0.f;
-    if (e < E) {
-        float u[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-        int64_t t = a + g;
-        for (; t + 28 < b; t += 32) {
-#pragma unroll
-            for (int i = 0; i < 8; ++i) u[i] += dz[(t + 4 * i) * E + e];
-        }
-        for (; t < b; t += 4) u[0] += dz[t * E + e];
-        acc = ((u[0] + u[1]) + (u[2] + u[3])) + ((u[4] + u[5]) + (u[6] + u[7]));
-    }
-    s_part[g][e] = acc;
+    if (g < G)
+        for (int64_t t = a + g; t < b; t += G) acc += dz[t * E + e];
+    s_part[threadIdx.x] = acc;
     __syncthreads();
-    if (g == 0 && e < E) part_db[(int64_t)c * E + e] = ((s_part[0][e] + s_part[1][e]) + s_part[2][e]) + s_part[3][e];
+    if (threadIdx.x < E) {
+        float sum = 0.f;
+        for (int q = 0; q < G; ++q) sum += s_part[q * E + threadIdx.x];
+        part_db[(int64_t)c * E + threadIdx.x] = sum;
+    }
 }
 
 // Partial dW_r = dlogits^T x and db over one chunk of RB_CH tokens of one party, for
