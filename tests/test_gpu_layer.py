@@ -78,6 +78,11 @@ SMALL = {
     "party4_bf16_T1024": lambda: mi.SHAPES[5].with_(T=1024),
     "all_experts_k_eq_E": lambda: mi.MoEShape("kE", 200, 256, 4, 256, 4, "bf16", seed=77),
     "one_token": lambda: mi.MoEShape("t1", 1, 128, 8, 128, 2, "bf16", seed=78),
+    # E % 4 != 0 (CUDA-core router forward), d % 256 != 0 (128-wide tiles; dX and dW1
+    # in separate launches), three parties of 233 tokens (router-gradient chunks end
+    # inside a 64-token block)
+    "odd_E6_d384_parties3": lambda: mi.MoEShape("o6", 699, 384, 6, 256, 2, "bf16", n_parties=3,
+                                                seed=79),
 }
 
 
