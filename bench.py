@@ -219,6 +219,19 @@ def run_reference(a):
     print(json.dumps(line))
 
 
+# --------------------------------------------------------------------------- ranks
+def max_over_ranks(vals, world: int, device: str = "cuda"):
+    """Element-wise maximum of `vals` over the ranks of the default process group (the
+    slowest replica sets the step time). Identity for a single process."""
+    if world <= 1:
+        return list(vals)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(v) for v in vals], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return t.tolist()
+
+
 # --------------------------------------------------------------------------- our arm
 def main():
     a = args_()
@@ -293,10 +306,7 @@ def main():
     ms_marked = statistics.mean([e["start"].elapsed_time(e["end"]) for e in evm])
     gms = statistics.mean([e["ffn_fwd_begin"].elapsed_time(e["ffn_fwd_end"]) +
                            e["ffn_bwd_begin"].elapsed_time(e["ffn_bwd_end"]) for e in evm])
-    if world > 1:
-        t = torch.tensor([ms, gms, ms_marked], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms, gms, ms_marked = t.tolist()
+    ms, gms, ms_marked = max_over_ranks([ms, gms, ms_marked], world)
     value = world * sh.T / (ms / 1e3)
 
     # e2e: host buffers in, host results out, through the same public calls
@@ -319,10 +329,7 @@ def main():
             e1.synchronize()
             times.append(e0.elapsed_time(e1))
         ems = statistics.mean(times)
-        if world > 1:
-            t = torch.tensor([ems], device="cuda")
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            ems = t.item()
+        ems = max_over_ranks([ems], world)[0]
         nb = 2 if sh.dtype == "bf16" else 4
         e2e = {"value": world * sh.T / (ems / 1e3), "unit": "tokens/s",
                "h2d_bytes_per_step": 2 * sh.T * sh.d_model * nb,
