@@ -344,11 +344,16 @@ def main():
     pk = peaks()
     gemm_flops = sh.gemm_flops()
     achieved = gemm_flops / (gms / 1e3) / 1e12
-    n_gemm = 6 + (6 if sh.n_shared else 0)
+    # expert-GEMM launches: GEMM1, GEMM2, then dA with dW2 and dX with dW1 (one launch
+    # each on the tensor cores; four on the CUDA cores)
+    n_gemm = (4 if sh.dtype == "bf16" else 6) + (6 if sh.n_shared else 0)
     traffic = gemm_traffic_record(sh)
     roofline = {"bound": "tensor", "kernel": "grouped_gemm_kernel (tcgen05, all expert GEMM launches)",
                 "achieved": achieved, "peak": pk["bf16_tflops"], "unit": "TFLOP/s",
                 "frac": achieved / pk["bf16_tflops"], "traffic": traffic,
+                "peak_sustained": pk["bf16_tflops_sustained"],
+                "frac_sustained": (achieved / pk["bf16_tflops_sustained"]
+                                   if pk["bf16_tflops_sustained"] else None),
                 "launches_per_step": n_gemm,
                 "peak_source": f"{pk['source']} bf16 burst"}
     mem_ms = ms_marked - gms  # both from the marked pass
