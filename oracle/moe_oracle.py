@@ -141,6 +141,57 @@ def dispatch_tables(idx, n_experts: int):
     return counts, offsets, slot_of, token_of
 
 
+def owner_of(e: int, n_parties: int) -> int:
+    """The party hosting expert e: round-robin over the parties (Sec. 3.1 item 2; R7)."""
+    return e % n_parties
+
+
+def owner_dispatch_tables(idx, n_experts: int, party_offsets):
+    """The dispatch grouped by receiving party: the layout of the cross-party sends of
+    Alg. 3 ("send h to the host of idx") when expert e lives on party owner(e).
+
+    group_expert[g] = the g-th expert in (owner, expert) order
+    counts_g, offsets_g, slot(t, j), token_of as dispatch_tables, with the expert
+      segments in that order: slot(t, j) = offsets_{pos(I_tj)} + #{t' < t : I_tj in I_t'}
+    send[s, o] = #{(t, j) : t in party s, owner(I_tj) = o}  (sends from s received by o;
+      tokens are party-contiguous, so inside a segment the rows of each source party are
+      contiguous and in party order)
+    """
+    idx = np.asarray(idx)
+    T, k = idx.shape
+    po = np.asarray(party_offsets, dtype=np.int64)
+    P = len(po) - 1
+    group_expert = sorted(range(n_experts), key=lambda e: (owner_of(e, P), e))
+    pos = np.empty(n_experts, np.int64)
+    for g, e in enumerate(group_expert):
+        pos[e] = g
+    counts = np.zeros(n_experts, np.int64)  # per segment g
+    for t in range(T):
+        for j in range(k):
+            counts[pos[idx[t, j]]] += 1
+    offsets = np.zeros(n_experts + 1, np.int64)
+    for g in range(n_experts):
+        offsets[g + 1] = offsets[g] + counts[g]
+    seen = np.zeros(n_experts, np.int64)
+    slot_of = np.empty((T, k), np.int64)
+    for t in range(T):
+        for j in range(k):
+            g = pos[idx[t, j]]
+            slot_of[t, j] = offsets[g] + seen[g]
+        for j in range(k):
+            seen[pos[idx[t, j]]] += 1
+    token_of = np.empty(T * k, np.int64)
+    for t in range(T):
+        for j in range(k):
+            token_of[slot_of[t, j]] = t
+    send = np.zeros((P, P), np.int64)
+    party = party_of_tokens(T, po)
+    for t in range(T):
+        for j in range(k):
+            send[party[t], owner_of(idx[t, j], P)] += 1
+    return np.asarray(group_expert, np.int64), counts, offsets, slot_of, token_of, send
+
+
 def party_counts(idx, n_experts: int, party_offsets) -> np.ndarray:
     """counts_{p,e}: how many of party p's (token, pick) pairs went to expert e."""
     po = np.asarray(party_offsets, dtype=np.int64)

@@ -116,6 +116,44 @@ def test_dispatch_tables_brute_force(T, E, k):
             assert (xp[slot_of[t, j]] == x[t]).all()
 
 
+@pytest.mark.parametrize("T,E,k,P", [(1, 1, 1, 1), (12, 4, 2, 2), (99, 8, 3, 3), (200, 32, 2, 4),
+                                      (60, 6, 2, 4)])
+def test_owner_dispatch_tables(T, E, k, P):
+    """Owner-grouped dispatch: segments in (owner = e mod P, expert) order, rows in token
+    order; pinned to a library lexsort of the (owner, expert, token) keys, to the plain
+    dispatch when P = 1, and to send counts recomputed from the permuted layout."""
+    rng = np.random.default_rng(T * 7 + E + k + P)
+    idx = np.stack([rng.permutation(E)[:k] for _ in range(T)]).astype(np.int32)
+    po = np.linspace(0, T, P + 1).astype(np.int64)
+    ge, counts, offsets, slot_of, token_of, send = mo.owner_dispatch_tables(idx, E, po)
+    # segment order: owners ascending, experts ascending inside an owner
+    assert sorted(ge.tolist(), key=lambda e: (e % P, e)) == ge.tolist()
+    assert sorted(ge.tolist()) == list(range(E))
+    # the permutation is a stable sort of the (t, j) entries by (owner, expert)
+    flat_e = idx.ravel().astype(np.int64)
+    flat_t = np.repeat(np.arange(T), k)
+    order = np.lexsort((flat_t, flat_e, flat_e % P))
+    assert (token_of == flat_t[order]).all()
+    assert (slot_of.ravel()[order] == np.arange(T * k)).all()
+    for g, e in enumerate(ge):  # segment g holds exactly expert e's rows
+        seg = slice(offsets[g], offsets[g + 1])
+        assert counts[g] == (flat_e == e).sum()
+        assert (idx[token_of[seg]] == e).any(axis=1).all()
+    # send counts: totals, per-source totals, and recomputed from the layout
+    assert send.sum() == T * k
+    assert (send.sum(axis=1) == np.diff(po) * k).all()
+    party = np.searchsorted(po, np.arange(T), side="right") - 1
+    re = np.zeros((P, P), np.int64)
+    for g, e in enumerate(ge):
+        for r in range(offsets[g], offsets[g + 1]):
+            re[party[token_of[r]], e % P] += 1
+    assert (re == send).all()
+    if P == 1:
+        c1, o1, s1, t1 = mo.dispatch_tables(idx, E)
+        assert (counts == c1).all() and (offsets == o1).all()
+        assert (slot_of == s1).all() and (token_of == t1).all()
+
+
 def test_combine_with_identity_experts():
     rng = np.random.default_rng(5)
     T, E, k, d = 40, 6, 3, 7
