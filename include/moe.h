@@ -125,6 +125,28 @@ moe_status moe_dispatch(const moe_config* cfg, const int32_t* topk_idx, const vo
                         void* workspace, size_t workspace_bytes, moe_stream_t stream);
 
 /*
+ * Owner-grouped dispatch: the layout of the cross-party sends of Alg. 3 ("send h to the
+ * host of idx") when expert e is hosted by party owner(e) = e mod P (round-robin,
+ * Sec. 3.1). As moe_dispatch, but the expert segments of x_perm are ordered by
+ * (owner, expert): every party's received rows are contiguous, and inside a segment the
+ * rows follow the token order (tokens are party-contiguous, so each source party's rows
+ * are contiguous and in party order).
+ *   group_expert [E] i32 out: the expert of segment g ((e mod P, e) order)
+ *   offsets [E+1] i32 out:    segment g holds rows [offsets[g], offsets[g+1])
+ *   slot_of, token_of, x_perm: as moe_dispatch, in this layout
+ *   send_counts [P,P] i32 out: (token, pick) pairs of source party s received by owner o
+ * The expert FFN calls take group_expert to find each segment's weights. P = 1 gives
+ * the expert-major layout of moe_dispatch. workspace: at least moe_workspace_size()
+ * bytes (also when T == 0). Returns MOE_ERR_DEVICE_CHECK (via moe_device_status) if an
+ * index is outside [0,E).
+ */
+moe_status moe_dispatch_owner(const moe_config* cfg, const int32_t* topk_idx, const void* x,
+                              const int32_t* party_offsets, int32_t* group_expert,
+                              int32_t* offsets, int32_t* slot_of, int32_t* token_of, void* x_perm,
+                              int32_t* send_counts, void* workspace, size_t workspace_bytes,
+                              moe_stream_t stream);
+
+/*
  * moe_dispatch without a workspace argument, for callers that cannot allocate device
  * memory: code whose host framework hands it only input and output buffers (an op or
  * plugin interface with no scratch), or that must not allocate while it runs (a
@@ -155,11 +177,14 @@ moe_status moe_dispatch_noalloc(const moe_config* cfg, const int32_t* topk_idx, 
  * Shared experts (all NULL when S == 0): x [T,d]; ws1 [S,2Fs,d]; ws2 [S,d,Fs];
  *   h_gu_sh [S,T,2Fs] out; act_sh [S,T,Fs] out; y_sh [S,T,d] out.
  * bf16: tcgen05 tensor-core GEMMs, fp32 accumulation in TMEM, bf16 outputs.
+ * group_expert [E] i32 (from moe_dispatch_owner) or NULL: segment g of x_perm (rows
+ *   [offsets[g], offsets[g+1])) belongs to expert group_expert[g] (NULL: to expert g).
  */
 moe_status moe_expert_ffn_fwd(const moe_config* cfg, const void* x_perm, const int32_t* offsets,
                               const void* w1, const void* w2, void* h_gu, void* act,
                               void* y_perm, const void* x, const void* ws1, const void* ws2,
-                              void* h_gu_sh, void* act_sh, void* y_sh, moe_stream_t stream);
+                              void* h_gu_sh, void* act_sh, void* y_sh,
+                              const int32_t* group_expert, moe_stream_t stream);
 
 /*
  * The weighted sum of Alg. 3: out_t = sum_j topk_w[t,j] * y_perm[slot_of[t*k+j]]
@@ -191,13 +216,15 @@ moe_status moe_combine_bwd(const moe_config* cfg, const void* dout, const void* 
  * Shared experts (NULL when S == 0): x [T,d], dout [T,d] (their dY), ws1, ws2,
  *   h_gu_sh, act_sh (forward), dh_sh [S,T,2Fs] out, dx_sh [S,T,d] out,
  *   dws1 [S,2Fs,d] out, dws2 [S,d,Fs] out.
+ * group_expert: as in moe_expert_ffn_fwd (dw1[e], dw2[e] are always expert e's).
  */
 moe_status moe_expert_ffn_bwd(const moe_config* cfg, const void* x_perm, const int32_t* offsets,
                               const void* w1, const void* w2, const void* h_gu, const void* act,
                               const void* dy_perm, void* dh, void* dx_perm, void* dw1, void* dw2,
                               const void* x, const void* dout, const void* ws1, const void* ws2,
                               const void* h_gu_sh, const void* act_sh, void* dh_sh, void* dx_sh,
-                              void* dws1, void* dws2, moe_stream_t stream);
+                              void* dws1, void* dws2, const int32_t* group_expert,
+                              moe_stream_t stream);
 
 /*
  * Backward of the gating function (the router is part of the party's local

@@ -66,10 +66,11 @@ _SIGS = {
     "moe_aux_loss": [_CFG] + [P] * 6,
     "moe_dispatch": [_CFG] + [P] * 7 + [ctypes.c_size_t, P],
     "moe_dispatch_noalloc": [_CFG] + [P] * 7,
-    "moe_expert_ffn_fwd": [_CFG] + [P] * 14,
+    "moe_dispatch_owner": [_CFG] + [P] * 10 + [ctypes.c_size_t, P],
+    "moe_expert_ffn_fwd": [_CFG] + [P] * 15,
     "moe_combine_fwd": [_CFG] + [P] * 6,
     "moe_combine_bwd": [_CFG] + [P] * 7,
-    "moe_expert_ffn_bwd": [_CFG] + [P] * 22,
+    "moe_expert_ffn_bwd": [_CFG] + [P] * 23,
     "moe_route_bwd": [_CFG] + [P] * 13 + [ctypes.c_size_t, P],
     "moe_dispatch_bwd": [_CFG] + [P] * 6,
     "moe_device_status": [P, ctypes.POINTER(ctypes.c_int32)],
@@ -186,10 +187,17 @@ def moe_dispatch_noalloc(cfg, topk_idx, x, offsets, slot_of, token_of, x_perm, s
           stream=stream)
 
 
+def moe_dispatch_owner(cfg, topk_idx, x, party_offsets, group_expert, offsets, slot_of, token_of,
+                       x_perm, send_counts, workspace, workspace_bytes, stream=None):
+    _call("moe_dispatch_owner", cfg, topk_idx, x, party_offsets, group_expert, offsets, slot_of,
+          token_of, x_perm, send_counts, workspace, int(workspace_bytes), stream=stream)
+
+
 def moe_expert_ffn_fwd(cfg, x_perm, offsets, w1, w2, h_gu, act, y_perm, x=None, ws1=None,
-                       ws2=None, h_gu_sh=None, act_sh=None, y_sh=None, stream=None):
+                       ws2=None, h_gu_sh=None, act_sh=None, y_sh=None, group_expert=None,
+                       stream=None):
     _call("moe_expert_ffn_fwd", cfg, x_perm, offsets, w1, w2, h_gu, act, y_perm, x, ws1, ws2,
-          h_gu_sh, act_sh, y_sh, stream=stream)
+          h_gu_sh, act_sh, y_sh, group_expert, stream=stream)
 
 
 def moe_combine_fwd(cfg, y_perm, topk_w, slot_of, y_sh, out, stream=None):
@@ -202,9 +210,11 @@ def moe_combine_bwd(cfg, dout, y_perm, topk_w, slot_of, dy_perm, dtopk_w, stream
 
 def moe_expert_ffn_bwd(cfg, x_perm, offsets, w1, w2, h_gu, act, dy_perm, dh, dx_perm, dw1, dw2,
                        x=None, dout=None, ws1=None, ws2=None, h_gu_sh=None, act_sh=None,
-                       dh_sh=None, dx_sh=None, dws1=None, dws2=None, stream=None):
+                       dh_sh=None, dx_sh=None, dws1=None, dws2=None, group_expert=None,
+                       stream=None):
     _call("moe_expert_ffn_bwd", cfg, x_perm, offsets, w1, w2, h_gu, act, dy_perm, dh, dx_perm,
-          dw1, dw2, x, dout, ws1, ws2, h_gu_sh, act_sh, dh_sh, dx_sh, dws1, dws2, stream=stream)
+          dw1, dw2, x, dout, ws1, ws2, h_gu_sh, act_sh, dh_sh, dx_sh, dws1, dws2, group_expert,
+          stream=stream)
 
 
 def moe_route_bwd(cfg, x, w_router, probs, topk_idx, topk_w, dtopk_w, aux_coef, party_offsets,

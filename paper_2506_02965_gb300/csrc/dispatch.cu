@@ -2,6 +2,8 @@
 // buffer), the gate-weighted combine of Alg. 3 and the backward of both (Alg. 5,
 // Sec. 3.2). All memory-bound: 16-byte vector loads/stores, one warp per token or
 // per permuted row, no floating-point atomics (every result is deterministic).
+#include <algorithm>
+
 #include "moe_common.cuh"
 #include "moe_internal.h"
 
@@ -10,37 +12,58 @@ namespace moe {
 constexpr int DCH = 128;  // tokens per dispatch chunk (one thread each)
 
 // Per chunk: how many of its (token, pick) pairs went to each expert. Also checks
-// that every index lies in [0, E) and that no token picks an expert twice.
+// that every index lies in [0, E) and that no token picks an expert twice. With `send`
+// (owner-grouped dispatch) it also adds each pair to send[party(t) * P + e mod P]
+// (integer additions: the totals do not depend on their order).
+constexpr int SEND_SMEM = 1024;  // P*P counters staged in shared memory up to this many
 __global__ void __launch_bounds__(DCH) chunk_count_kernel(const int32_t* __restrict__ idx,
                                                           int64_t T, int E, int k,
-                                                          int32_t* chunk_counts) {
+                                                          int32_t* chunk_counts,
+                                                          const int32_t* __restrict__ po, int P,
+                                                          int32_t* send) {
     pdl_begin();
     __shared__ int s_cnt[64];
+    __shared__ int s_send[SEND_SMEM];
+    const bool send_smem = send && P * P <= SEND_SMEM;
     for (int i = threadIdx.x; i < E; i += blockDim.x) s_cnt[i] = 0;
+    if (send_smem)
+        for (int i = threadIdx.x; i < P * P; i += blockDim.x) s_send[i] = 0;
     __syncthreads();
     const int64_t t = (int64_t)blockIdx.x * DCH + threadIdx.x;
     if (t < T) {
+        const int src = send ? party_of(po, P, t) : 0;
         for (int j = 0; j < k; ++j) {
             const int e = idx[t * k + j];
             bool ok = (e >= 0 && e < E);
             for (int jj = 0; jj < j; ++jj) ok = ok && (idx[t * k + jj] != e);
-            if (ok) atomicAdd(&s_cnt[e], 1);
-            else record_status(MOE_ERR_DEVICE_CHECK);
+            if (ok) {
+                atomicAdd(&s_cnt[e], 1);
+                if (send_smem) atomicAdd(&s_send[src * P + e % P], 1);
+                else if (send) atomicAdd(&send[src * P + e % P], 1);
+            } else {
+                record_status(MOE_ERR_DEVICE_CHECK);
+            }
         }
     }
     __syncthreads();
     for (int i = threadIdx.x; i < E; i += blockDim.x)
         chunk_counts[(int64_t)blockIdx.x * E + i] = s_cnt[i];
+    if (send_smem)
+        for (int i = threadIdx.x; i < P * P; i += blockDim.x)
+            if (s_send[i]) atomicAdd(&send[i], s_send[i]);
 }
 
 // Per chunk: offsets (written by chunk 0), the chunk's base row inside each expert
 // segment, and the stable rank of each pick among the chunk's picks of that expert
-// (a bit per token and expert, counted with popc).
+// (a bit per token and expert, counted with popc). The expert segments follow in
+// (e mod Pown, e) order: expert order for Pown = 1, owner-grouped for Pown = P (chunk 0
+// then also writes group_expert[g] = the expert of segment g).
 __global__ void __launch_bounds__(DCH) slot_kernel(const int32_t* __restrict__ idx,
                                                    const int32_t* __restrict__ chunk_counts,
                                                    int64_t T, int E, int k, int nchunks,
                                                    int32_t* offsets, int32_t* slot_of,
-                                                   int32_t* token_of) {
+                                                   int32_t* token_of, int Pown,
+                                                   int32_t* group_expert) {
     pdl_begin();
     __shared__ int s_pre[64];
     __shared__ int s_tot[64];
@@ -67,11 +90,16 @@ __global__ void __launch_bounds__(DCH) slot_kernel(const int32_t* __restrict__ i
     for (int i = threadIdx.x; i < 64 * (DCH / 32); i += blockDim.x) (&s_bits[0][0])[i] = 0u;
     __syncthreads();
     if (threadIdx.x == 0) {
-        int run = 0;
-        for (int e = 0; e < E; ++e) {
-            if (c == 0) offsets[e] = run;
-            s_base[e] = run + s_pre[e];
-            run += s_tot[e];
+        int run = 0, g = 0;
+        for (int o = 0; o < Pown; ++o) {
+            for (int e = o; e < E; e += Pown, ++g) {
+                if (c == 0) {
+                    offsets[g] = run;
+                    if (group_expert) group_expert[g] = e;
+                }
+                s_base[e] = run + s_pre[e];
+                run += s_tot[e];
+            }
         }
         if (c == 0) offsets[E] = run;
     }
@@ -341,19 +369,27 @@ size_t dispatch_workspace(int64_t T, int E) {
 
 cudaError_t launch_dispatch(const int32_t* topk_idx, const void* x, int64_t T, int d, int E, int k,
                             bool bf16, int32_t* offsets, int32_t* slot_of, int32_t* token_of,
-                            void* x_perm, void* ws, cudaStream_t s) {
-    const int nch = (int)((T + DCH - 1) / DCH);
+                            void* x_perm, void* ws, cudaStream_t s, const int32_t* po, int P,
+                            int32_t* group_expert, int32_t* send) {
+    const bool owner = send != nullptr;
+    const int nch = (int)std::max<int64_t>(owner ? 1 : 0, (T + DCH - 1) / DCH);
     int32_t* cc = (int32_t*)ws;
-    if (T == 0) {
+    cudaError_t e;
+    if (owner) {
+        if ((e = cudaMemsetAsync(send, 0, sizeof(int32_t) * P * P, s)) != cudaSuccess) return e;
+    } else if (T == 0) {
         return cudaMemsetAsync(offsets, 0, sizeof(int32_t) * (E + 1), s);
     }
-    (void)launch_pdl(chunk_count_kernel, dim3(nch), dim3(DCH), 0, s, topk_idx, T, E, k, cc);
-    cudaError_t e = cudaGetLastError();
+    (void)launch_pdl(chunk_count_kernel, dim3(nch), dim3(DCH), 0, s, topk_idx, T, E, k, cc, po,
+                     owner ? P : 1, send);
+    e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    (void)launch_pdl(slot_kernel, dim3(nch), dim3(DCH), 0, s, topk_idx, cc, T, E, k, nch, offsets, slot_of, token_of);
+    (void)launch_pdl(slot_kernel, dim3(nch), dim3(DCH), 0, s, topk_idx, cc, T, E, k, nch, offsets,
+                     slot_of, token_of, owner ? P : 1, group_expert);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     const int64_t TK = T * k;
+    if (TK == 0) return cudaSuccess;
     const unsigned blocks = (unsigned)((TK + 7) / 8);
     if (bf16)
         (void)launch_pdl(gather_kernel<__nv_bfloat16>, dim3(blocks), dim3(256), 0, s, (const __nv_bfloat16*)x, token_of, TK, T,
@@ -461,10 +497,12 @@ cudaError_t launch_dispatch_noalloc(const int32_t* topk_idx, const void* x, int6
     const int nch = (int)((T + DCH - 1) / DCH);
     if ((int64_t)nch * E > kNoAllocScratchInts) return cudaErrorInvalidValue;
     if (T == 0) return cudaMemsetAsync(offsets, 0, sizeof(int32_t) * (E + 1), s);
-    (void)launch_pdl(chunk_count_kernel, dim3(nch), dim3(DCH), 0, s, topk_idx, T, E, k, cc);
+    (void)launch_pdl(chunk_count_kernel, dim3(nch), dim3(DCH), 0, s, topk_idx, T, E, k, cc,
+                     (const int32_t*)nullptr, 1, (int32_t*)nullptr);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    (void)launch_pdl(slot_kernel, dim3(nch), dim3(DCH), 0, s, topk_idx, cc, T, E, k, nch, offsets, slot_of, token_of);
+    (void)launch_pdl(slot_kernel, dim3(nch), dim3(DCH), 0, s, topk_idx, cc, T, E, k, nch, offsets,
+                     slot_of, token_of, 1, (int32_t*)nullptr);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     const int64_t TK = T * k;

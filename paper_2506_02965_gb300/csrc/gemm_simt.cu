@@ -64,7 +64,7 @@ __global__ void __launch_bounds__(256) gemm_m_simt_kernel(GemmMArgs p) {
     const int F = (p.epi == EPI_SWIGLU_FWD) ? N / 2 : N;
     const int n0 = blockIdx.x * (p.epi == EPI_SWIGLU_FWD ? SB_N / 2 : SB_N);
     const float* A = (const float*)p.a;
-    const float* B = (const float*)p.b + (int64_t)g * p.b_group_elems;
+    const float* B = (const float*)p.b + (int64_t)(p.group_expert ? p.group_expert[g] : g) * p.b_group_elems;
     const int Nb = (p.epi == EPI_SWIGLU_FWD) ? N : N;  // rows of B viewed as [Nb, K]
     float acc[4][4] = {};
     for (int k0 = 0; k0 < K; k0 += SB_K) {
@@ -191,7 +191,7 @@ __global__ void __launch_bounds__(256) gemm_k_simt_kernel(GemmKArgs p) {
         }
         __syncthreads();
     }
-    float* out = (float*)p.out + (int64_t)g * M * N;
+    float* out = (float*)p.out + (int64_t)(p.group_expert ? p.group_expert[g] : g) * M * N;
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
         const int m = m0 + ty * 4 + i;

@@ -46,6 +46,7 @@ struct Params {
     int Mout;    // output rows per group (K-variable)
     int F;       // SwiGLU inner size (SWIGLU epilogues)
     int64_t b_group_rows;  // rows of B's 2D view per group (M-variable)
+    const int32_t* gexp;   // group -> expert of its weights / weight gradient, or null
     void* out0;
     void* out1;
     const void* aux;
@@ -316,6 +317,8 @@ struct Tile {
     int k_iters;
     int last_rows;      // K-var: valid contraction rows in the last k-block (1..64)
     bool dw;            // a tile of the second (K-variable) problem of a fused launch
+    int we;             // expert whose weights (M-variable) or weight gradient (K-variable)
+                        // the tile uses: group_expert[g], or g
 };
 
 // ------------------------------------------------------------------------ router epilogue
@@ -490,6 +493,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                 const int tn2 = p2.N / BN;
                 ti.dw = true;
                 ti.g = g;
+                ti.we = p2.gexp ? p2.gexp[g] : g;
                 ti.m0 = (l2 / tn2) * BM;
                 ti.n0 = (l2 % tn2) * BN;
                 const int64_t r0 = p2.offsets[g], nrows = p2.offsets[g + 1] - r0;
@@ -506,6 +510,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         const int local = t - s_tile_start[g];
         const int mt = local / tiles_n, nt = local % tiles_n;
         ti.g = g;
+        ti.we = p.gexp ? p.gexp[g] : g;
         ti.m0 = mt * BMP + (int)rank * BM;
         ti.n0 = nt * ((EPI == EPI_SWIGLU_FWD) ? 128 : BN);
         int64_t r0, nrows, a0, b0, o0;
@@ -655,7 +660,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                     if (EPI == EPI_SWIGLU_FWD) {
                         // 128 gate rows then 128 up rows of the same features; in a pair the
                         // leader holds the gate half and the peer the up half
-                        const int64_t r = (int64_t)ti.g * p.b_group_rows + ti.n0;
+                        const int64_t r = (int64_t)ti.we * p.b_group_rows + ti.n0;
                         if constexpr (PAIR) {
                             load(sb, &tmB, fb, k0, (int)(r + (rank ? p.F : 0)));
                         } else {
@@ -663,9 +668,9 @@ __global__ void __launch_bounds__(THREADS, 1)
                             load(sb + 128 * 128, &tmB, fb, k0, (int)(r + p.F));
                         }
                     } else if (!B_MN) {
-                        load(sb, &tmB, fb, k0, (int)((int64_t)ti.g * p.b_group_rows + ti.n0 + rank * BNL));
+                        load(sb, &tmB, fb, k0, (int)((int64_t)ti.we * p.b_group_rows + ti.n0 + rank * BNL));
                     } else {
-                        const int64_t krow = (VAR_K || dw) ? (ti.b_row + k0) : ((int64_t)ti.g * p.b_group_rows + k0);
+                        const int64_t krow = (VAR_K || dw) ? (ti.b_row + k0) : ((int64_t)ti.we * p.b_group_rows + k0);
                         const CUtensorMap* mB = dw ? &tmB2 : &tmB;
 #pragma unroll
                         for (int i = 0; i < BNL / 64; ++i)
@@ -829,7 +834,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             const int wrow0 = ti.m0 + q * 32;
             const bool full_box = wrow0 + 32 <= ti.mvalid;
             const bool dwt = DW2 && ti.dw;
-            const int64_t grow0 = (VAR_K || dwt) ? (int64_t)ti.g * (dwt ? p2.Mout : p.Mout) + wrow0
+            const int64_t grow0 = (VAR_K || dwt) ? (int64_t)ti.we * (dwt ? p2.Mout : p.Mout) + wrow0
                                                  : ti.out_row + wrow0;
             const uint32_t tbase = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
             // write NOUT rows of 32 values each: staged + TMA when the whole box is valid
@@ -859,7 +864,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                 // second problem: a bf16 weight-gradient tile, [Mout, N] per group
                 if (!wait_bar(tfull_bar(acc), acc_phase)) break;
                 fence_after();
-                __nv_bfloat16* out = (__nv_bfloat16*)p2.out0 + (int64_t)ti.g * p2.Mout * p2.N + (int64_t)m * p2.N;
+                __nv_bfloat16* out = (__nv_bfloat16*)p2.out0 + (int64_t)ti.we * p2.Mout * p2.N + (int64_t)m * p2.N;
 #pragma unroll 1
                 for (int c = 0; c < BN; c += 32) {
                     float y[32];
@@ -980,7 +985,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                 } else {
                     __nv_bfloat16* out;
                     if (VAR_K)
-                        out = (__nv_bfloat16*)p.out0 + (int64_t)ti.g * p.Mout * p.N + (int64_t)m * p.N;
+                        out = (__nv_bfloat16*)p.out0 + (int64_t)ti.we * p.Mout * p.N + (int64_t)m * p.N;
                     else
                         out = (__nv_bfloat16*)p.out0 + (ti.out_row + m) * (int64_t)p.N;
 #pragma unroll 1
@@ -1197,6 +1202,7 @@ cudaError_t launch_gemm_m(const GemmMArgs& g, bool bf16, cudaStream_t s) {
     p.out1 = g.out1;
     p.aux = g.aux;
     p.wait_ns = g_wait_ns;
+    p.gexp = g.group_expert;
     // A rows in the 2D view: OFFSETS -> all routed rows; UNIFORM -> groups * stride (or rows)
     const int64_t a_rows = g.rows.offsets ? (int64_t)g.rows.rows
                                           : std::max<int64_t>(g.rows.rows, (int64_t)(g.G - 1) * g.rows.a_stride + g.rows.rows);
@@ -1271,6 +1277,7 @@ cudaError_t launch_gemm_k(const GemmKArgs& g, bool bf16, cudaStream_t s) {
     p.Mout = g.M;
     p.out0 = g.out;
     p.wait_ns = g_wait_ns;
+    p.gexp = g.group_expert;
     const int64_t rows_a = g.rows.offsets ? (int64_t)g.rows.rows
                                           : std::max<int64_t>(g.rows.rows, (int64_t)(g.G - 1) * g.rows.a_stride + g.rows.rows);
     const int64_t rows_b = g.rows.offsets ? (int64_t)g.rows.rows
@@ -1313,6 +1320,7 @@ cudaError_t launch_gemm_mk(const GemmMArgs& g, const GemmKArgs& k, cudaStream_t 
     p.out1 = g.out1;
     p.aux = g.aux;
     p.wait_ns = g_wait_ns;
+    p.gexp = g.group_expert;
     p.b_group_rows = g.b_rows ? g.b_rows : g.K;
     const int64_t a_rows = (int64_t)g.rows.rows, o_rows = a_rows;
     CUtensorMap ma, mb, mo0, mo1;
@@ -1334,6 +1342,7 @@ cudaError_t launch_gemm_mk(const GemmMArgs& g, const GemmKArgs& k, cudaStream_t 
     p2.Mout = k.M;
     p2.out0 = k.out;
     p2.wait_ns = g_wait_ns;
+    p2.gexp = k.group_expert;
     CUtensorMap ma2, mb2, mo2;
     if (!make_map(&ma2, k.a, k.M, (int64_t)k.rows.rows, 64)) return cudaErrorInvalidValue;
     if (!make_map(&mb2, k.b, k.N, (int64_t)k.rows.rows, 64)) return cudaErrorInvalidValue;

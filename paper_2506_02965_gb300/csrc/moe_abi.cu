@@ -264,6 +264,36 @@ moe_status moe_dispatch(const moe_config* cfg, const int32_t* topk_idx, const vo
                        "moe_dispatch");
 }
 
+moe_status moe_dispatch_owner(const moe_config* cfg, const int32_t* topk_idx, const void* x,
+                              const int32_t* party_offsets, int32_t* group_expert,
+                              int32_t* offsets, int32_t* slot_of, int32_t* token_of, void* x_perm,
+                              int32_t* send_counts, void* workspace, size_t workspace_bytes,
+                              moe_stream_t stream) {
+    moe_status st = check_cfg(cfg);
+    if (st) return st;
+    if ((st = check_parties(cfg, party_offsets))) return st;
+    REQUIRE(group_expert);
+    REQUIRE(offsets);
+    REQUIRE(send_counts);
+    REQUIRE(workspace);
+    const size_t need = dispatch_workspace(std::max<int64_t>(cfg->T, 1), cfg->n_experts);
+    if (workspace_bytes < need)
+        return fail(MOE_ERR_INVALID_ARG, "workspace of %zu bytes < %zu needed", workspace_bytes, need);
+    if (cfg->T > 0) {
+        REQUIRE(topk_idx);
+        REQUIRE_VEC(x);
+        REQUIRE(slot_of);
+        REQUIRE(token_of);
+        REQUIRE_VEC(x_perm);
+    }
+    return cuda_status(launch_dispatch(topk_idx, x, cfg->T, cfg->d_model, cfg->n_experts,
+                                       cfg->top_k, cfg->dtype == MOE_BF16, offsets, slot_of,
+                                       token_of, x_perm, workspace, (cudaStream_t)stream,
+                                       cfg->n_parties > 1 ? party_offsets : nullptr,
+                                       cfg->n_parties, group_expert, send_counts),
+                       "moe_dispatch_owner");
+}
+
 moe_status moe_dispatch_noalloc(const moe_config* cfg, const int32_t* topk_idx, const void* x,
                                 int32_t* offsets, int32_t* slot_of, int32_t* token_of,
                                 void* x_perm, moe_stream_t stream) {
@@ -292,7 +322,8 @@ moe_status moe_dispatch_noalloc(const moe_config* cfg, const int32_t* topk_idx, 
 moe_status moe_expert_ffn_fwd(const moe_config* cfg, const void* x_perm, const int32_t* offsets,
                               const void* w1, const void* w2, void* h_gu, void* act, void* y_perm,
                               const void* x, const void* ws1, const void* ws2, void* h_gu_sh,
-                              void* act_sh, void* y_sh, moe_stream_t stream) {
+                              void* act_sh, void* y_sh, const int32_t* group_expert,
+                              moe_stream_t stream) {
     moe_status st = check_cfg(cfg);
     if (st) return st;
     const bool bf16 = cfg->dtype == MOE_BF16;
@@ -317,6 +348,7 @@ moe_status moe_expert_ffn_fwd(const moe_config* cfg, const void* x_perm, const i
     cudaStream_t s = (cudaStream_t)stream;
     // routed experts: [G|U] = Xp W1^T with SwiGLU epilogue, then Y = A W2^T
     GemmMArgs g1{};
+    g1.group_expert = group_expert;
     g1.G = E;
     g1.rows = GroupRows{offsets, (int)TK, 0, 0, 0};
     g1.a = x_perm;
@@ -330,6 +362,7 @@ moe_status moe_expert_ffn_fwd(const moe_config* cfg, const void* x_perm, const i
     g1.out1 = act;
     if ((st = cuda_status(launch_gemm_m(g1, bf16, s), "expert gemm1"))) return st;
     GemmMArgs g2{};
+    g2.group_expert = group_expert;
     g2.G = E;
     g2.rows = GroupRows{offsets, (int)TK, 0, 0, 0};
     g2.a = act;
@@ -344,6 +377,7 @@ moe_status moe_expert_ffn_fwd(const moe_config* cfg, const void* x_perm, const i
     if (S) {
         const int Fs = cfg->d_ff_shared;
         GemmMArgs h1 = g1;
+        h1.group_expert = nullptr;  // shared experts: one group per expert
         h1.G = S;
         h1.rows = GroupRows{nullptr, (int)T, 0, 0, T};
         h1.a = x;
@@ -354,6 +388,7 @@ moe_status moe_expert_ffn_fwd(const moe_config* cfg, const void* x_perm, const i
         h1.out1 = act_sh;
         if ((st = cuda_status(launch_gemm_m(h1, bf16, s), "shared gemm1"))) return st;
         GemmMArgs h2 = g2;
+        h2.group_expert = nullptr;  // shared experts: one group per expert
         h2.G = S;
         h2.rows = GroupRows{nullptr, (int)T, T, 0, T};
         h2.a = act_sh;
@@ -406,7 +441,8 @@ moe_status moe_expert_ffn_bwd(const moe_config* cfg, const void* x_perm, const i
                               const void* dy_perm, void* dh, void* dx_perm, void* dw1, void* dw2,
                               const void* x, const void* dout, const void* ws1, const void* ws2,
                               const void* h_gu_sh, const void* act_sh, void* dh_sh, void* dx_sh,
-                              void* dws1, void* dws2, moe_stream_t stream) {
+                              void* dws1, void* dws2, const int32_t* group_expert,
+                              moe_stream_t stream) {
     moe_status st = check_cfg(cfg);
     if (st) return st;
     const bool bf16 = cfg->dtype == MOE_BF16;
@@ -451,6 +487,7 @@ moe_status moe_expert_ffn_bwd(const moe_config* cfg, const void* x_perm, const i
     }
     // dA = dY W2 with the SwiGLU-backward epilogue -> dH
     GemmMArgs a{};
+    a.group_expert = group_expert;
     a.G = E;
     a.rows = GroupRows{offsets, (int)TK, 0, 0, 0};
     a.a = dy_perm;
@@ -464,6 +501,7 @@ moe_status moe_expert_ffn_bwd(const moe_config* cfg, const void* x_perm, const i
     a.out0 = dh;
     // dXp = dH W1
     GemmMArgs b{};
+    b.group_expert = group_expert;
     b.G = E;
     b.rows = GroupRows{offsets, (int)TK, 0, 0, 0};
     b.a = dh;
@@ -476,6 +514,7 @@ moe_status moe_expert_ffn_bwd(const moe_config* cfg, const void* x_perm, const i
     b.out0 = dx_perm;
     // dW2[e] = dY_e^T A_e ; dW1[e] = dH_e^T Xp_e
     GemmKArgs w2g{};
+    w2g.group_expert = group_expert;
     w2g.G = E;
     w2g.rows = GroupRows{offsets, (int)TK, 0, 0, 0};
     w2g.a = dy_perm;
@@ -484,6 +523,7 @@ moe_status moe_expert_ffn_bwd(const moe_config* cfg, const void* x_perm, const i
     w2g.N = F;
     w2g.out = dw2;
     GemmKArgs w1g{};
+    w1g.group_expert = group_expert;
     w1g.G = E;
     w1g.rows = GroupRows{offsets, (int)TK, 0, 0, 0};
     w1g.a = dh;
@@ -524,6 +564,7 @@ moe_status moe_expert_ffn_bwd(const moe_config* cfg, const void* x_perm, const i
     }
     if (S) {
         GemmMArgs sa = a;
+        sa.group_expert = nullptr;  // shared experts: one group per expert
         sa.G = S;
         sa.rows = GroupRows{nullptr, (int)T, 0, 0, T};
         sa.a = dout;
@@ -534,6 +575,7 @@ moe_status moe_expert_ffn_bwd(const moe_config* cfg, const void* x_perm, const i
         sa.out0 = dh_sh;
         if ((st = cuda_status(launch_gemm_m(sa, bf16, s), "shared dA gemm"))) return st;
         GemmMArgs sb = b;
+        sb.group_expert = nullptr;  // shared experts: one group per expert
         sb.G = S;
         sb.rows = GroupRows{nullptr, (int)T, T, 0, T};
         sb.a = dh_sh;
@@ -543,6 +585,7 @@ moe_status moe_expert_ffn_bwd(const moe_config* cfg, const void* x_perm, const i
         sb.out0 = dx_sh;
         if ((st = cuda_status(launch_gemm_m(sb, bf16, s), "shared dX gemm"))) return st;
         GemmKArgs sw2 = w2g;
+        sw2.group_expert = nullptr;  // shared experts: one group per expert
         sw2.G = S;
         sw2.rows = GroupRows{nullptr, (int)T, 0, T, 0};
         sw2.a = dout;
@@ -551,6 +594,7 @@ moe_status moe_expert_ffn_bwd(const moe_config* cfg, const void* x_perm, const i
         sw2.out = dws2;
         if ((st = cuda_status(launch_gemm_k(sw2, bf16, s), "shared dW2 gemm"))) return st;
         GemmKArgs sw1 = w1g;
+        sw1.group_expert = nullptr;  // shared experts: one group per expert
         sw1.G = S;
         sw1.rows = GroupRows{nullptr, (int)T, T, 0, 0};
         sw1.a = dh_sh;

@@ -55,7 +55,9 @@ cudaError_t route_status(cudaStream_t s, int* code);
 size_t dispatch_workspace(int64_t T, int E);
 cudaError_t launch_dispatch(const int32_t* topk_idx, const void* x, int64_t T, int d, int E, int k,
                             bool bf16, int32_t* offsets, int32_t* slot_of, int32_t* token_of,
-                            void* x_perm, void* ws, cudaStream_t s);
+                            void* x_perm, void* ws, cudaStream_t s,
+                            const int32_t* po = nullptr, int P = 1,
+                            int32_t* group_expert = nullptr, int32_t* send = nullptr);
 cudaError_t launch_combine_fwd(const void* y_perm, const float* topk_w, const int32_t* slot_of,
                                const void* y_sh, int S, int64_t T, int d, int k, bool bf16,
                                void* out, cudaStream_t s);
@@ -102,6 +104,8 @@ struct GemmMArgs {
     int N, K;
     int b_rows;  // MN-major B: rows of one group's [K, N] view when they are fewer than K
                  // (the rows past them multiply zero columns of A); 0 means K
+    const int32_t* group_expert;  // device [G]: the weights of group g are group_expert[g]'s
+                                  // (owner-grouped layout); null: group g's
     int epi;
     // EPI_SWIGLU_FWD: out0 = h_gu [rows, 2F] (G at cols [0,F), U at [F,2F)),
     //                 out1 = act [rows, F]; N = 2F (B holds gate rows then up rows).
@@ -125,6 +129,7 @@ struct GemmKArgs {
     // stored transposed, out + (g*E + e)*M + m = C_g[m, e] for e < E.
     int epi = EPI_STORE;
     int E = 0;
+    const int32_t* group_expert = nullptr;  // device [G]: group g's output is group_expert[g]'s
 };
 
 cudaError_t launch_gemm_m(const GemmMArgs& g, bool bf16, cudaStream_t s);

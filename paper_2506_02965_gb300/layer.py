@@ -19,8 +19,11 @@ from . import _lib as L
 
 
 class MoELayer:
-    def __init__(self, shape, device: str = "cuda"):
+    def __init__(self, shape, device: str = "cuda", owner_grouped=None):
+        """owner_grouped: lay the permuted rows out by owner party (expert e hosted by
+        party e mod P, moe_dispatch_owner) instead of by expert; default: when P > 1."""
         self.shape = sh = shape
+        self.owner_grouped = (sh.n_parties > 1) if owner_grouped is None else bool(owner_grouped)
         self.device = device
         self.dt = torch.bfloat16 if sh.dtype == "bf16" else torch.float32
         self.cfg = L.make_config(sh.T, sh.d_model, sh.n_experts, sh.d_ff, sh.top_k, sh.n_parties,
@@ -47,6 +50,10 @@ class MoELayer:
         self.counts = z(P, E, dtype=i32)
         self.aux_loss, self.aux_coef = z(P, dtype=f32), z(P, E, dtype=f32)
         self.offsets = z(E + 1, dtype=i32)
+        # owner-grouped layout: the expert of each segment, and the (source party ->
+        # owner party) pair counts of the sends
+        self.group_expert = z(E, dtype=i32) if self.owner_grouped else None
+        self.send_counts = z(P, P, dtype=i32) if self.owner_grouped else None
         self.slot_of, self.token_of = z(TK, dtype=i32), z(TK, dtype=i32)
         self.x_perm = z(TK, d)
         self.h_gu, self.act, self.y_perm = z(TK, 2 * F), z(TK, F), z(TK, d)
@@ -113,12 +120,17 @@ class MoELayer:
                        stream=self.side)
         aux_done = torch.cuda.Event()
         aux_done.record(self.side)
-        L.moe_dispatch(c, self.topk_idx, self.x, self.offsets, self.slot_of, self.token_of,
-                       self.x_perm, self.workspace, self.ws_bytes, stream=main)
+        if self.owner_grouped:
+            L.moe_dispatch_owner(c, self.topk_idx, self.x, self.party_offsets, self.group_expert,
+                                 self.offsets, self.slot_of, self.token_of, self.x_perm,
+                                 self.send_counts, self.workspace, self.ws_bytes, stream=main)
+        else:
+            L.moe_dispatch(c, self.topk_idx, self.x, self.offsets, self.slot_of, self.token_of,
+                           self.x_perm, self.workspace, self.ws_bytes, stream=main)
         mark("ffn_fwd_begin")
         L.moe_expert_ffn_fwd(c, self.x_perm, self.offsets, self.w1, self.w2, self.h_gu, self.act,
                              self.y_perm, self.x, self.ws1, self.ws2, self.h_gu_sh, self.act_sh,
-                             self.y_sh, stream=main)
+                             self.y_sh, group_expert=self.group_expert, stream=main)
         mark("ffn_fwd_end")
         L.moe_combine_fwd(c, self.y_perm, self.topk_w, self.slot_of, self.y_sh, self.out,
                           stream=main)
@@ -144,7 +156,8 @@ class MoELayer:
         L.moe_expert_ffn_bwd(c, self.x_perm, self.offsets, self.w1, self.w2, self.h_gu, self.act,
                              self.dy_perm, self.dh, self.dx_perm, self.dw1, self.dw2, self.x,
                              self.dout, self.ws1, self.ws2, self.h_gu_sh, self.act_sh, self.dh_sh,
-                             self.dx_sh, self.dws1, self.dws2, stream=main)
+                             self.dx_sh, self.dws1, self.dws2, group_expert=self.group_expert,
+                             stream=main)
         mark("ffn_bwd_end")
         main.wait_event(join)
         L.moe_dispatch_bwd(c, self.dx_perm, self.slot_of, self.dx_router, self.dx_sh, self.dx,

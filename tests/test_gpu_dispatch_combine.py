@@ -61,6 +61,40 @@ def test_dispatch_tables_bit_exact(L, T, E, k, pattern, dtype):
     assert (xp.float().cpu().numpy() == x[tok]).all()  # a copy: bit-exact
 
 
+OWNER_CASES = [(1000, 8, 2, 2, "uniform"), (999, 32, 2, 3, "uniform"), (333, 6, 2, 4, "skewed"),
+               (4096, 64, 6, 8, "uniform"), (512, 16, 2, 1, "uniform"), (0, 8, 2, 2, "uniform")]
+
+
+@pytest.mark.parametrize("T,E,k,P,pattern", OWNER_CASES)
+def test_owner_dispatch_tables_bit_exact(L, T, E, k, P, pattern):
+    """Owner-grouped dispatch: segment order, offsets, slots, token map, the permuted
+    copy and the per-(source, owner) send counts against the oracle, bit for bit (P = 1
+    gives the expert-major tables; T = 0 still writes the order and zero counts)."""
+    d = 256
+    idx = picks(T, E, k, pattern, seed=T + E + P) if T else np.zeros((0, k), np.int32)
+    sh = mi.MoEShape("o", T, d, E, 256, k, "bf16", n_parties=P)
+    cfg = cfg_of(L, sh)
+    x = mi.bf16_round(np.random.default_rng(2).standard_normal((max(T, 1), d)).astype(np.float32))[:T]
+    po = np.asarray([T * p // P for p in range(P + 1)], np.int32)
+    ws = L.moe_workspace_size(cfg)
+    wsb = torch.empty(ws, dtype=torch.uint8, device="cuda")
+    ge, offsets = empty((E,), torch.int32), empty((E + 1,), torch.int32)
+    slot_of, token_of = empty((max(T * k, 1),), torch.int32), empty((max(T * k, 1),), torch.int32)
+    xp, send = empty((max(T * k, 1), d), torch.bfloat16), empty((P, P), torch.int32)
+    L.moe_dispatch_owner(cfg, dev(idx, torch.int32) if T else None, dev(x, torch.bfloat16) if T else None,
+                         dev(po, torch.int32), ge, offsets, slot_of if T else None,
+                         token_of if T else None, xp if T else None, send, wsb, ws)
+    assert status(L) == 0
+    rge, counts, off, slot, tok, rsend = mo.owner_dispatch_tables(idx, E, po)
+    assert (ints(ge) == rge).all()
+    assert (ints(offsets) == off).all()
+    assert (ints(send) == rsend).all()
+    if T:
+        assert (ints(slot_of) == slot.ravel()).all()
+        assert (ints(token_of) == tok).all()
+        assert (xp.float().cpu().numpy() == x[tok]).all()
+
+
 def test_dispatch_detects_bad_index(L):
     T, E, k, d = 300, 8, 2, 128
     idx = picks(T, E, k, "uniform")

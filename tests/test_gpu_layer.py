@@ -41,18 +41,28 @@ def full_compare(lay, inp, sh):
     # integer work: bit-exact
     assert (ints(lay.topk_idx) == fwd["topk_idx"]).all()
     assert (ints(lay.counts) == fwd["party_counts"]).all()
-    assert (ints(lay.offsets) == fwd["offsets"]).all()
-    assert (ints(lay.slot_of) == fwd["slot_of"].ravel()).all()
-    assert (ints(lay.token_of) == fwd["token_of"]).all()
-    assert (np64(lay.x_perm) == fwd["x_perm"]).all()
+    rows = np.arange(sh.T * sh.top_k)  # GPU permuted row -> oracle (expert-major) row
+    if lay.owner_grouped:
+        ge, _, off, slot, tok, send = mo.owner_dispatch_tables(fwd["topk_idx"], sh.n_experts,
+                                                              inp["party_offsets"])
+        assert (ints(lay.group_expert) == ge).all()
+        assert (ints(lay.send_counts) == send).all()
+        rows = np.empty_like(rows)
+        rows[slot.ravel()] = fwd["slot_of"].ravel()
+    else:
+        off, slot, tok = fwd["offsets"], fwd["slot_of"], fwd["token_of"]
+    assert (ints(lay.offsets) == off).all()
+    assert (ints(lay.slot_of) == slot.ravel()).all()
+    assert (ints(lay.token_of) == tok).all()
+    assert (np64(lay.x_perm) == fwd["x_perm"][rows]).all()
     errs = {}
     for name, gpu, ref in [
         ("probs", lay.probs, fwd["probs"]), ("topk_w", lay.topk_w, fwd["topk_w"]),
-        ("h_gu", lay.h_gu, fwd["h_gu"]), ("act", lay.act, fwd["act"]),
-        ("y_perm", lay.y_perm, fwd["y_perm"]), ("out", lay.out, fwd["out"]),
+        ("h_gu", lay.h_gu, fwd["h_gu"][rows]), ("act", lay.act, fwd["act"][rows]),
+        ("y_perm", lay.y_perm, fwd["y_perm"][rows]), ("out", lay.out, fwd["out"]),
         ("aux_loss", lay.aux_loss, fwd["aux_loss"]), ("aux_coef", lay.aux_coef, fwd["aux_coef"]),
-        ("dy_perm", lay.dy_perm, bwd["dy_perm"]), ("dtopk_w", lay.dtopk_w, bwd["dtopk_w"]),
-        ("dh", lay.dh, bwd["dh"]), ("dx_perm", lay.dx_perm, bwd["dx_perm"]),
+        ("dy_perm", lay.dy_perm, bwd["dy_perm"][rows]), ("dtopk_w", lay.dtopk_w, bwd["dtopk_w"]),
+        ("dh", lay.dh, bwd["dh"][rows]), ("dx_perm", lay.dx_perm, bwd["dx_perm"][rows]),
         ("dw1", lay.dw1, bwd["dw1"]), ("dw2", lay.dw2, bwd["dw2"]),
         ("dlogits", lay.dlogits, bwd["dlogits"]), ("dw_router", lay.dw_router, bwd["dw_router"]),
         ("dbias", lay.dbias, bwd["dbias"]), ("dx_router", lay.dx_router, bwd["dx_router"]),
@@ -134,6 +144,34 @@ def test_step_from_host_buffers_matches_device_step(L):
         assert torch.equal(hloss, ref.aux_loss.cpu()), i
         assert torch.equal(lay.dw1, ref.dw1), i
     assert status(L) == 0
+
+
+@pytest.mark.parametrize("sh", [mi.SHAPES[5].with_(T=1024), mi.SHAPES[3].with_(T=512, n_parties=2),
+                                mi.SHAPES[2].with_(T=1000)], ids=["party4", "fine_P2", "mid_P1"])
+def test_owner_grouped_layout_gives_the_same_results(L, sh):
+    """The layer with its permuted rows grouped by owner party (moe_dispatch_owner, the
+    expert GEMMs told each segment's expert) equals the expert-major layer bit for bit:
+    every expert sees the same rows in the same order. The send counts match the picks."""
+    inp = mi.make_inputs(sh)
+    a, b = MoELayer(sh, owner_grouped=True), MoELayer(sh, owner_grouped=False)
+    for lay in (a, b):
+        lay.load(inp)
+        lay.step()
+    torch.cuda.synchronize()
+    assert status(L) == 0
+    for n in ("out", "dx", "dw1", "dw2", "dw_router", "dbias", "dlogits", "dtopk_w", "aux_loss",
+              "topk_idx", "counts"):
+        assert torch.equal(getattr(a, n), getattr(b, n)), n
+    if sh.n_shared:
+        for n in ("dws1", "dws2", "y_sh"):
+            assert torch.equal(getattr(a, n), getattr(b, n)), n
+    idx = ints(a.topk_idx)
+    P = sh.n_parties
+    part = mo.party_of_tokens(sh.T, inp["party_offsets"])
+    ref = np.zeros((P, P), np.int64)
+    np.add.at(ref, (np.repeat(part, sh.top_k), idx.ravel() % P), 1)
+    assert (ints(a.send_counts) == ref).all()
+    assert (ints(a.group_expert) == sorted(range(sh.n_experts), key=lambda e: (e % P, e))).all()
 
 
 def test_layer_empty_batch(L):
