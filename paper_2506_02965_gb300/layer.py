@@ -78,6 +78,9 @@ class MoELayer:
         self.side = torch.cuda.Stream(device=device)
         # host<->device copies that overlap the passes (step_host)
         self.copy_stream = torch.cuda.Stream(device=device)
+        # device->host copies of pipelined passes (run_host), and their second buffer set
+        self.d2h_stream = torch.cuda.Stream(device=device)
+        self._io_alt = None
         self.ws_bytes = L.moe_workspace_size(self.cfg)
         self.workspace = torch.empty(max(self.ws_bytes, 16), dtype=torch.uint8, device=device)
 
@@ -201,6 +204,72 @@ class MoELayer:
             hdx.copy_(self.dx, non_blocking=True)
             hloss.copy_(self.aux_loss, non_blocking=True)
         main.wait_event(out_back)
+
+    def run_host(self, batches, stream=None):
+        """Several fwd+bwd passes fed from host memory, pipelined: the uploads of pass
+        i+1 and the downloads of pass i-1 run on two copy streams beside the kernels of
+        pass i. ``batches`` is a sequence of (hx, hdout, hout, hdx, hloss) host tensors as
+        in ``step_host`` (pinned); pass i reads hx, hdout of its own tuple and writes its
+        hout, hdx, hloss. x, dout, out, dx and the aux loss alternate between two device
+        buffer sets; the weight gradients (dw1, dw2, dw_router, dbias) are those of the
+        last pass. Returns once every pass is queued; synchronize before reading."""
+        main = stream if stream is not None else torch.cuda.current_stream()
+        if self._io_alt is None:
+            self._io_alt = tuple(torch.empty_like(t) for t in self._io_tensors())
+        sets = (self._io_tensors(), self._io_alt)
+        h2d, d2h = self.copy_stream, self.d2h_stream
+        n = len(batches)
+        start = torch.cuda.Event()
+        start.record(main)  # earlier work on this stream owns set 0 until here
+        h2d.wait_event(start)
+        d2h.wait_event(start)
+        done = [None] * n      # pass i finished reading its inputs and writing its outputs
+        arrived = [None] * n   # pass i's inputs are on the device
+        fetched = [None] * n   # pass i's outputs are on the host
+
+        def upload(i):
+            hx, hdout = batches[i][0], batches[i][1]
+            x, dout = sets[i % 2][0], sets[i % 2][1]
+            if i >= 2:
+                h2d.wait_event(done[i - 2])
+            with torch.cuda.stream(h2d):
+                x.copy_(hx, non_blocking=True)
+                dout.copy_(hdout, non_blocking=True)
+            arrived[i] = torch.cuda.Event()
+            arrived[i].record(h2d)
+
+        try:
+            if n:
+                upload(0)
+            for i in range(n):
+                if i + 1 < n:
+                    upload(i + 1)
+                self._set_io(sets[i % 2])
+                main.wait_event(arrived[i])
+                if i >= 2:
+                    main.wait_event(fetched[i - 2])  # set i % 2's outputs are on the host
+                self.forward(main)
+                self.backward(main)
+                done[i] = torch.cuda.Event()
+                done[i].record(main)
+                d2h.wait_event(done[i])
+                hout, hdx, hloss = batches[i][2], batches[i][3], batches[i][4]
+                with torch.cuda.stream(d2h):
+                    hout.copy_(self.out, non_blocking=True)
+                    hdx.copy_(self.dx, non_blocking=True)
+                    hloss.copy_(self.aux_loss, non_blocking=True)
+                fetched[i] = torch.cuda.Event()
+                fetched[i].record(d2h)
+        finally:
+            self._set_io(sets[0])
+        for ev in fetched[-2:]:
+            main.wait_event(ev)  # later work on this stream may reuse both sets
+
+    def _io_tensors(self):
+        return (self.x, self.dout, self.out, self.dx, self.aux_loss)
+
+    def _set_io(self, t):
+        self.x, self.dout, self.out, self.dx, self.aux_loss = t
 
     def kernels_per_step(self) -> int:
         """CUDA kernels this library launches per step (memsets not counted):

@@ -146,6 +146,40 @@ def test_step_from_host_buffers_matches_device_step(L):
     assert status(L) == 0
 
 
+def test_pipelined_host_passes_match_device_steps(L):
+    """run_host: five passes with different inputs, uploads and downloads overlapping the
+    neighbouring passes' kernels on two copy streams and two device buffer sets; every
+    pass's out, dx and aux loss equal a device-resident step on the same inputs, bit for
+    bit, and the weight gradients are the last pass's. A copy that raced a pass, or a
+    buffer set reused too early, would change some pass's results."""
+    sh = mi.SHAPES[2].with_(T=1024)
+    lay, ref = MoELayer(sh), MoELayer(sh)
+    lay.load(mi.make_inputs(sh))
+    ref.load(mi.make_inputs(sh))
+    n = 5
+    batches = []
+    for i in range(n):
+        inp = mi.make_inputs(sh.with_(seed=sh.seed + 200 + i), with_weights=False)
+        hx = torch.from_numpy(inp["x"]).to(lay.dt).pin_memory()
+        hd = torch.from_numpy(inp["dout"]).to(lay.dt).pin_memory()
+        batches.append((hx, hd, torch.empty_like(hx).pin_memory(), torch.empty_like(hx).pin_memory(),
+                        torch.full((sh.n_parties,), float("nan")).pin_memory()))
+    x0 = lay.x
+    lay.run_host(batches)
+    torch.cuda.synchronize()
+    for i, (hx, hd, ho, hdx, hloss) in enumerate(batches):
+        ref.x.copy_(hx)
+        ref.dout.copy_(hd)
+        ref.step()
+        torch.cuda.synchronize()
+        assert torch.equal(ho, ref.out.cpu()), i
+        assert torch.equal(hdx, ref.dx.cpu()), i
+        assert torch.equal(hloss, ref.aux_loss.cpu()), i
+    assert torch.equal(lay.dw1, ref.dw1) and torch.equal(lay.dw_router, ref.dw_router)
+    assert lay.x is x0  # the first buffer set is current again
+    assert status(L) == 0
+
+
 @pytest.mark.parametrize("sh", [mi.SHAPES[5].with_(T=1024), mi.SHAPES[3].with_(T=512, n_parties=2),
                                 mi.SHAPES[2].with_(T=1000)], ids=["party4", "fine_P2", "mid_P1"])
 def test_owner_grouped_layout_gives_the_same_results(L, sh):
