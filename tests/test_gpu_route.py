@@ -48,11 +48,20 @@ def test_route_from_logits_bit_exact(L, T, E, k, P, norm):
     assert_close("topk_w", w, mo.gate_weights(p, ref_idx, norm), 1e-6)
 
 
-@pytest.mark.parametrize("which,T", [(1, None), (2, None), (5, 2048), (4, 1024), (3, 1024)])
-def test_route_matches_oracle(L, which, T):
+@pytest.mark.parametrize("which,T,extra", [
+    (1, None, {}), (2, None, {}), (5, 2048, {}), (4, 1024, {}), (3, 1024, {}),
+    # 128 tiles, more than one per CTA on some SMs
+    (2, 16384, {}),
+    # d = 384 (6 k-blocks), three parties of 233 tokens: ragged tiles that end mid-party
+    (2, 699, {"d_model": 384, "n_experts": 8, "n_parties": 3}),
+    # E = 32 (N = 32), a single partial tile
+    (2, 77, {"n_experts": 32})])
+def test_route_matches_oracle(L, which, T, extra):
+    """The tensor-core gating (router GEMM with the gating in its epilogue) against the
+    fp64 oracle: logits within the accumulation tolerance, picks and counts exact."""
     sh = mi.SHAPES[which]
     if T:
-        sh = sh.with_(T=T)
+        sh = sh.with_(T=T, **extra)
     sh = sh.with_(seed=seeds.decided_seed(sh))
     inp = mi.make_inputs(sh, with_weights=False)
     dt = torch.bfloat16 if sh.dtype == "bf16" else torch.float32
