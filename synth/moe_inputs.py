@@ -174,3 +174,38 @@ def make_route_logits(T: int, E: int, seed: int, tie_every: int = 7) -> np.ndarr
         lo = max(0, E // 2 - 2)
         z[t, lo:lo + min(4, E)] = z[t, lo]
     return z
+
+
+# ----------------------------------------------------------------------------- training
+def party_schedule(n_parties: int, epochs: int, seed: int) -> list:
+    """The order in which the parties take their turns: one seeded random permutation
+    of 0..n-1 per epoch (the RandomPermutation of Alg. 1), drawn from one generator."""
+    rng = np.random.default_rng(seed)
+    return [rng.permutation(n_parties).astype(np.int64).tolist() for _ in range(epochs)]
+
+
+def train_batches(shape: MoEShape, n_parties: int, n_batches: int, seed: int) -> list:
+    """Each party's private data D_i: ``n_batches`` batches of shape.T tokens, as
+    [(x, y), ...] per party. x ~ N(0,1); the regression target is a fixed random
+    linear map of x, y = x R / sqrt(d) with R ~ N(0,1) [d,d] shared by all parties
+    (one teacher, so the parties' objectives agree). float32, bf16-rounded for bf16
+    shapes. Draw order: R, then party by party, batch by batch, x then nothing else."""
+    rng = np.random.default_rng(seed)
+    d = shape.d_model
+    R = rng.standard_normal((d, d), dtype=np.float32) / np.float32(np.sqrt(d))
+    out = []
+    for _ in range(n_parties):
+        mine = []
+        for _ in range(n_batches):
+            x = _normal(rng, (shape.T, d), 1.0, shape.dtype)
+            y = (x @ R).astype(np.float32)
+            mine.append((x, bf16_round(y) if shape.dtype == "bf16" else y))
+        out.append(mine)
+    return out
+
+
+def train_init(shape: MoEShape, n_parties: int, seed: int) -> dict:
+    """The common initialization of Alg. 1: every party's router W_r[i] and the expert
+    pool W1, W2, drawn as in ``make_inputs`` for a shape with n_parties routers."""
+    inp = make_inputs(shape.with_(n_parties=n_parties, T=n_parties), seed=seed)
+    return {"w_router": inp["w_router"], "w1": inp["w1"], "w2": inp["w2"]}
