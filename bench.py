@@ -50,6 +50,10 @@ def args_():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
+    ap.add_argument("--train", action="store_true",
+                    help="time Alg. 1 training steps (layer + MSE loss + SGD) instead")
+    ap.add_argument("--parties", type=int, default=4, help="parties taking turns (--train)")
+    ap.add_argument("--lr", type=float, default=0.05, help="SGD step (--train)")
     return ap.parse_args()
 
 
@@ -237,10 +241,79 @@ def max_over_ranks(vals, world: int, device: str = "cuda"):
 
 
 # --------------------------------------------------------------------------- our arm
+def train_bench(a):
+    """Alg. 1 on one GPU: the parties take turns (a seeded permutation per epoch), one
+    batch of the workload's T tokens per turn; a step is the layer's forward and
+    backward, the MSE loss and the SGD updates of the active party's gating and of the
+    experts its batch called. Inputs resident in HBM; no L2 flush (each step streams
+    the expert weights, their gradients and the updated weights, several times L2)."""
+    import torch
+    from paper_2506_02965_gb300 import _lib as L
+    from paper_2506_02965_gb300.train import RoundRobinTrainer
+
+    torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
+    base = mi.shape_by_name(a.workload)
+    sh = base.with_(n_parties=1, n_shared=0, d_ff_shared=0)
+    n = max(1, a.parties)
+    tr = RoundRobinTrainer(sh, n, lr=a.lr)
+    tr.load(mi.train_init(sh, n, seed=sh.seed))
+    tdt = tr.layer.dt
+    batches = [[(torch.from_numpy(x).to("cuda", tdt), torch.from_numpy(y).to("cuda", tdt))
+                for x, y in mine] for mine in mi.train_batches(sh, n, 1, seed=sh.seed + 1)]
+    w_epochs = max(1, -(-max(3, a.warmup) // n))
+    t_epochs = max(1, -(-a.steps // n))
+    sched = mi.party_schedule(n, w_epochs + t_epochs, seed=sh.seed + 2)
+    tr.run(batches, sched[:w_epochs], 1)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    _, log = tr.run(batches, sched[w_epochs:], 1)
+    e1.record()
+    torch.cuda.synchronize()
+    tr.layer.check_status()
+    steps = t_epochs * n
+    ms = e0.elapsed_time(e1) / steps
+    # the SGD updates alone (counts of the last batch), for their HBM fraction
+    lay, E, d, F = tr.layer, sh.n_experts, sh.d_model, sh.d_ff
+    called = int((lay.counts > 0).sum().item())
+    nb = 2 if sh.dtype == "bf16" else 4
+    # per element: read w (or the fp32 master) and dw, write w (and the master)
+    per_elem = (4 + nb + 4 + nb) if tr.master else 3 * nb
+    sgd_bytes = per_elem * (called * 3 * F * d + E * d)
+    g0, g1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    reps = 20
+    g0.record()
+    for _ in range(reps):  # lr = 0: the same traffic, parameters unchanged
+        L.moe_sgd_update(tr.w_router[0], lay.dw_router, 1, E * d, None, 0.0, tr.dtype,
+                         w_master=tr.m_router[0] if tr.master else None)
+        L.moe_sgd_update(lay.w1, lay.dw1, E, 2 * F * d, lay.counts, 0.0, tr.dtype, w_master=tr.m1)
+        L.moe_sgd_update(lay.w2, lay.dw2, E, d * F, lay.counts, 0.0, tr.dtype, w_master=tr.m2)
+    g1.record()
+    torch.cuda.synchronize()
+    sgd_ms = g0.elapsed_time(g1) / reps
+    pk = peaks()
+    losses = log.cpu().numpy()
+    line = {"metric": "Alg. 1 training step (MoE layer fwd+bwd + MSE + SGD) tokens/s on 1 GB300",
+            "value": sh.T / (ms / 1e3), "unit": "tokens/s", "n_gpus": 1, "steps": steps,
+            "warmup": w_epochs * n, "ms_per_step": ms, "higher_is_better": True,
+            "dtype": sh.dtype, "data": "synthetic (seeded numpy PCG64, regression on a fixed random teacher)",
+            "config": {"workload": f"{workload_desc(sh)}, {n} parties taking turns, B=1, SGD lr={a.lr}"
+                                    + (", fp32 master weights" if tr.master else ""),
+                       "l2": "not flushed: every step streams the weights and their gradients (> L2)"},
+            "sgd": {"ms_per_step": sgd_ms, "bytes": sgd_bytes, "achieved_gbs": sgd_bytes / sgd_ms / 1e6,
+                    "peak_gbs": pk["hbm_gbs"], "frac": sgd_bytes / sgd_ms / 1e6 / pk["hbm_gbs"]},
+            "loss_first_last": [float(losses[0].sum()), float(losses[-1].sum())],
+            "gpu_launches": steps * tr.kernels_per_step()}
+    print(json.dumps(line), flush=True)
+
+
 def main():
     a = args_()
     if a.impl == "reference":
         run_reference(a)
+        return
+    if a.train:
+        train_bench(a)
         return
     import torch
     import torch.distributed as dist

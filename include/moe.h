@@ -261,6 +261,39 @@ moe_status moe_dispatch_bwd(const moe_config* cfg, const void* dx_perm, const in
                             const void* dx_router, const void* dx_sh, void* dx,
                             moe_stream_t stream);
 
+/*
+ * Training step of Alg. 1 around the layer (toy block: the layer output is the block
+ * output). The loss of the batch, Loss(h, y) of Alg. 1, read as mean-squared error:
+ *   loss[0] = sum_t ||out_t - target_t||^2 / (2T)          (fp32, device out)
+ *   dout    = (out - target) / T                            [T,d] dtype out
+ * out, target [T,d] dtype (cfg->dtype). fp32 arithmetic; the reduction runs in a fixed
+ * order (the same bits on every call). workspace: device scratch of at least
+ * moe_workspace_size(cfg) bytes (only its first 2 KB are used here).
+ * Errors: MOE_ERR_INVALID_ARG for NULL pointers or a short workspace. T == 0 writes 0.
+ */
+moe_status moe_mse_loss(const moe_config* cfg, const void* out, const void* target, float* loss,
+                        void* dout, void* workspace, size_t workspace_bytes, moe_stream_t stream);
+
+/*
+ * One SGD step on a parameter stored as n_groups groups of group_elems elements (an
+ * expert stack [E, ...] or one party's router slice): the updates of Alg. 1, where
+ * only the active party's gating (BackwardLocal, Alg. 4) and the experts its batch
+ * called (BackwardExpert, Alg. 6) change and nothing is broadcast. For every group g
+ * with group_counts[g] > 0 (every group when group_counts is NULL):
+ *   w_master == NULL:  w[g] <- w[g] - lr * dw[g]
+ *   w_master != NULL:  w_master[g] <- w_master[g] - lr * dw[g];  w[g] <- w_master[g]
+ * w, dw [n_groups * group_elems] of dtype, device memory, updated in place; w_master
+ * (optional) fp32 [n_groups * group_elems] device memory, the master copy of w for
+ * bf16 training (updates below the bf16 spacing accumulate there); group_counts
+ * [n_groups] int32 device memory or NULL (e.g. the per-expert counts moe_route wrote
+ * for a one-party batch). fp32 arithmetic (one fused multiply-add), rounded to dtype.
+ * A group that is not called is neither read nor written.
+ * Errors: MOE_ERR_INVALID_ARG for negative sizes, more than 65535 groups, an unknown
+ * dtype, a non-finite lr or NULL w / dw with work to do.
+ */
+moe_status moe_sgd_update(void* w, const void* dw, float* w_master, int64_t n_groups, int64_t group_elems,
+                          const int32_t* group_counts, float lr, moe_dtype dtype, moe_stream_t stream);
+
 /* Synchronises `stream`, returns the first error code any kernel recorded since the
  * last call (MOE_OK if none) in *code and clears it. */
 moe_status moe_device_status(moe_stream_t stream, int32_t* code /* HOST out */);

@@ -74,7 +74,8 @@ def train_step(params, party: int, x, y, shape, lr: float):
     """One batch of Alg. 1's inner loop for party ``party``: forward, loss, backward,
     the router update (BackwardLocal) and the called experts' updates (BackwardExpert).
     ``shape`` describes the batch (T tokens, one party). Returns the new parameters
-    and a record: total loss, MSE, per-expert counts, gradients, updated parties."""
+    and a record: total loss, MSE, aux loss, per-expert counts, the smallest top-(k+1)
+    logit gap of the batch, gradients, updated parties."""
     inp = _layer_inputs(params, party, x)
     loss, mse, dout, fwd = batch_loss(params, party, x, y, shape)
     bwd = mo.layer_backward(inp, shape, fwd, dout=dout, with_aux=True)
@@ -85,7 +86,8 @@ def train_step(params, party: int, x, y, shape, lr: float):
     new["w2"] = sgd_groups(params["w2"], bwd["dw2"], lr, counts)
     n = np.asarray(params["w_router"]).shape[0]
     owners = {int(e) % n for e in np.nonzero(counts > 0)[0]}
-    rec = {"party": party, "loss": loss, "mse": mse, "counts": counts,
+    rec = {"party": party, "loss": loss, "mse": mse, "aux": float(fwd["aux_loss"][0]), "counts": counts,
+           "min_margin": float(mo.top_margin(fwd["logits"], shape.top_k).min()),
            "dw_router": bwd["dw_router"][0], "dw1": bwd["dw1"], "dw2": bwd["dw2"],
            "updated_parties": sorted(owners | {party})}
     return new, rec

@@ -76,6 +76,8 @@ _SIGS = {
     "moe_device_status": [P, ctypes.POINTER(ctypes.c_int32)],
     "moe_set_wait_limit_ns": [ctypes.c_uint64],
     "moe_set_gemm_pairs": [ctypes.c_int],
+    "moe_mse_loss": [_CFG] + [P] * 5 + [ctypes.c_size_t, P],
+    "moe_sgd_update": [P, P, P, ctypes.c_int64, ctypes.c_int64, P, ctypes.c_float, ctypes.c_int, P],
 }
 for _n, _a in _SIGS.items():
     f = getattr(_lib, _n)
@@ -198,6 +200,15 @@ def moe_expert_ffn_fwd(cfg, x_perm, offsets, w1, w2, h_gu, act, y_perm, x=None, 
                        stream=None):
     _call("moe_expert_ffn_fwd", cfg, x_perm, offsets, w1, w2, h_gu, act, y_perm, x, ws1, ws2,
           h_gu_sh, act_sh, y_sh, group_expert, stream=stream)
+
+
+def moe_mse_loss(cfg, out, target, loss, dout, workspace, workspace_bytes, stream=None):
+    _call("moe_mse_loss", cfg, out, target, loss, dout, workspace, workspace_bytes, stream=stream)
+
+
+def moe_sgd_update(w, dw, n_groups, group_elems, group_counts, lr, dtype, w_master=None, stream=None):
+    _check(_lib.moe_sgd_update(_ptr(w), _ptr(dw), _ptr(w_master), int(n_groups), int(group_elems),
+                               _ptr(group_counts), float(lr), int(dtype), _stream(stream)), "moe_sgd_update")
 
 
 def moe_combine_fwd(cfg, y_perm, topk_w, slot_of, y_sh, out, stream=None):

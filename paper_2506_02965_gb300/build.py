@@ -17,7 +17,7 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libmoe.so")
-SOURCES = ["route.cu", "dispatch.cu", "gemm_simt.cu", "gemm_tc.cu", "moe_abi.cu"]
+SOURCES = ["route.cu", "dispatch.cu", "gemm_simt.cu", "gemm_tc.cu", "train.cu", "moe_abi.cu"]
 HEADERS = ["moe_common.cuh", "moe_internal.h"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",

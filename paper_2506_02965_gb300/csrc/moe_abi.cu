@@ -153,8 +153,9 @@ moe_status moe_workspace_size(const moe_config* cfg, size_t* bytes) {
     moe_status st = check_cfg(cfg);
     if (st) return st;
     REQUIRE(bytes);
-    *bytes = std::max(dispatch_workspace(cfg->T, cfg->n_experts),
-                      route_bwd_workspace(cfg->T, cfg->n_parties, cfg->n_experts, cfg->d_model));
+    *bytes = std::max(std::max(dispatch_workspace(cfg->T, cfg->n_experts),
+                               route_bwd_workspace(cfg->T, cfg->n_parties, cfg->n_experts, cfg->d_model)),
+                      mse_workspace_bytes());
     return MOE_OK;
 }
 
@@ -670,6 +671,40 @@ moe_status moe_dispatch_bwd(const moe_config* cfg, const void* dx_perm, const in
                                                cfg->T, cfg->d_model, cfg->top_k,
                                                cfg->dtype == MOE_BF16, dx, (cudaStream_t)stream),
                        "moe_dispatch_bwd");
+}
+
+moe_status moe_mse_loss(const moe_config* cfg, const void* out, const void* target, float* loss,
+                        void* dout, void* workspace, size_t workspace_bytes, moe_stream_t stream) {
+    moe_status st = check_cfg(cfg);
+    if (st) return st;
+    REQUIRE(loss);
+    if (cfg->T == 0)
+        return cuda_status(cudaMemsetAsync(loss, 0, sizeof(float), (cudaStream_t)stream), "moe_mse_loss");
+    REQUIRE(out);
+    REQUIRE(target);
+    REQUIRE(dout);
+    REQUIRE(workspace);
+    if (workspace_bytes < mse_workspace_bytes())
+        return fail(MOE_ERR_INVALID_ARG, "workspace_bytes %zu < %zu", workspace_bytes, mse_workspace_bytes());
+    return cuda_status(launch_mse_loss(out, target, cfg->T, cfg->d_model, cfg->dtype == MOE_BF16, loss, dout,
+                                       workspace, (cudaStream_t)stream),
+                       "moe_mse_loss");
+}
+
+moe_status moe_sgd_update(void* w, const void* dw, float* w_master, int64_t n_groups, int64_t group_elems,
+                          const int32_t* group_counts, float lr, moe_dtype dtype, moe_stream_t stream) {
+    if (n_groups < 0 || group_elems < 0)
+        return fail(MOE_ERR_INVALID_ARG, "negative size (n_groups=%lld, group_elems=%lld)",
+                    (long long)n_groups, (long long)group_elems);
+    if (n_groups > 65535) return fail(MOE_ERR_INVALID_ARG, "n_groups=%lld > 65535", (long long)n_groups);
+    if (dtype != MOE_F32 && dtype != MOE_BF16) return fail(MOE_ERR_INVALID_ARG, "unknown dtype %d", (int)dtype);
+    if (!(lr == lr) || lr - lr != 0.0f) return fail(MOE_ERR_INVALID_ARG, "lr is not finite");
+    if (n_groups == 0 || group_elems == 0) return MOE_OK;
+    REQUIRE(w);
+    REQUIRE(dw);
+    return cuda_status(launch_sgd_update(w, dw, w_master, n_groups, group_elems, group_counts, lr, dtype == MOE_BF16,
+                                         (cudaStream_t)stream),
+                       "moe_sgd_update");
 }
 
 moe_status moe_device_status(moe_stream_t stream, int32_t* code) {

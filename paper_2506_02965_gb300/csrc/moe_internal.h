@@ -148,4 +148,11 @@ cudaError_t simt_status(cudaStream_t s, int* code);
 cudaError_t launch_gemm_m_simt(const GemmMArgs& g, cudaStream_t s);
 cudaError_t launch_gemm_k_simt(const GemmKArgs& g, cudaStream_t s);
 
+// training step around the layer (train.cu)
+cudaError_t launch_sgd_update(void* w, const void* dw, float* master, int64_t n_groups, int64_t group_elems,
+                              const int32_t* counts, float lr, bool bf16, cudaStream_t s);
+size_t mse_workspace_bytes();
+cudaError_t launch_mse_loss(const void* out, const void* y, int64_t T, int d, bool bf16, float* loss,
+                            void* dout, void* workspace, cudaStream_t s);
+
 }  // namespace moe

@@ -101,6 +101,28 @@ def test_null_and_misaligned_pointers_rejected_on_host(L):
         L.moe_set_wait_limit_ns(0)
 
 
+def test_training_calls_check_arguments_on_host(L):
+    """moe_sgd_update and moe_mse_loss reject bad arguments before any device work."""
+    cases = [((16, 16, -1, 8, None, 0.1, L.MOE_BF16), "negative size"),
+             ((16, 16, 70000, 8, None, 0.1, L.MOE_BF16), "65535"),
+             ((16, 16, 2, 8, None, float("nan"), L.MOE_F32), "lr"),
+             ((16, 16, 2, 8, None, float("inf"), L.MOE_F32), "lr"),
+             ((16, 16, 2, 8, None, 0.1, 7), "dtype"),
+             ((None, 16, 2, 8, None, 0.1, L.MOE_F32), "w is NULL")]
+    for args, frag in cases:
+        with pytest.raises(L.MoEError) as ei:
+            L.moe_sgd_update(*args, stream=0)
+        assert ei.value.status == L.MOE_ERR_INVALID_ARG and frag in L.moe_last_error(), frag
+    L.moe_sgd_update(None, None, 0, 8, None, 0.1, L.MOE_F32, stream=0)  # nothing to do: OK
+    cfg = L.make_config(256, 256, 8, 256, 2)
+    with pytest.raises(L.MoEError):
+        L.moe_mse_loss(cfg, 16, 16, 16, 16, 16, 8, stream=0)
+    assert "workspace_bytes" in L.moe_last_error()
+    with pytest.raises(L.MoEError):
+        L.moe_mse_loss(cfg, 16, None, 16, 16, 16, 4096, stream=0)
+    assert "target is NULL" in L.moe_last_error()
+
+
 def test_binding_refuses_to_load_without_library(L, monkeypatch):
     monkeypatch.setattr(L, "LIB_PATH", "/nonexistent/libmoe.so")
     with pytest.raises(ImportError):
