@@ -424,9 +424,11 @@ def main():
     pk = peaks()
     gemm_flops = sh.gemm_flops()
     achieved = gemm_flops / (gms / 1e3) / 1e12
-    # expert-GEMM launches: GEMM1, GEMM2, then dA with dW2 and dX with dW1 (one launch
-    # each on the tensor cores; four on the CUDA cores)
-    n_gemm = (4 if sh.dtype == "bf16" else 6) + (6 if sh.n_shared else 0)
+    # expert-GEMM launches: GEMM1, GEMM2 (+2 for shared experts), then the backward's as
+    # the library reports them (dA with dW2 in one launch, dX as CTA pairs beside dW1 on
+    # the tensor cores by default; four on the CUDA cores; shared experts' four)
+    from paper_2506_02965_gb300 import _lib as L
+    n_gemm = 2 + L.moe_expert_ffn_bwd_kernels(lay.cfg) + (2 if sh.n_shared else 0)
     traffic = gemm_traffic_record(sh)
     roofline = {"bound": "tensor", "kernel": "grouped_gemm_kernel (tcgen05, all expert GEMM launches)",
                 "achieved": achieved, "peak": pk["bf16_tflops"], "unit": "TFLOP/s",

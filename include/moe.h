@@ -186,6 +186,12 @@ moe_status moe_expert_ffn_fwd(const moe_config* cfg, const void* x_perm, const i
                               void* h_gu_sh, void* act_sh, void* y_sh,
                               const int32_t* group_expert, moe_stream_t stream);
 
+/* Number of CUDA kernels one moe_expert_ffn_bwd call with this configuration launches
+ * (host only, no device work): per weight, the input-gradient GEMM and the weight
+ * gradient in one persistent launch, or in two (CTA-pair tiles, moe_set_gemm_pairs,
+ * and the fp32 path), plus four for the shared experts; 0 GEMMs when T*k == 0. */
+moe_status moe_expert_ffn_bwd_kernels(const moe_config* cfg, int32_t* count /* HOST out */);
+
 /*
  * The weighted sum of Alg. 3: out_t = sum_j topk_w[t,j] * y_perm[slot_of[t*k+j]]
  * (+ sum_s y_sh[s,t] when S > 0, shared experts enter with weight 1).
@@ -309,8 +315,9 @@ moe_status moe_set_wait_limit_ns(uint64_t ns);
  * as few tiles share the SMs, so a launch with few tiles loses to its last round.
  *   MOE_PAIRS_OFF  (0): single-CTA tiles everywhere;
  *   MOE_PAIRS_ALL  (1): pair tiles for every such GEMM;
- *   MOE_PAIRS_AUTO (2, default): pair tiles where a launch has at least four rounds of
- *                   them and its epilogue is not the SwiGLU backward (which, not the
+ *   MOE_PAIRS_AUTO (2, default): pair tiles for the input-gradient GEMM dX = dH W1
+ *                   (contraction 2F) and wherever a launch has at least four rounds
+ *                   of them, except under the SwiGLU backward epilogue (which, not the
  *                   operand feed, bounds the dA GEMM).
  * Results agree up to fp32 summation order. Any other mode: MOE_ERR_INVALID_ARG. */
 enum { MOE_PAIRS_OFF = 0, MOE_PAIRS_ALL = 1, MOE_PAIRS_AUTO = 2 };

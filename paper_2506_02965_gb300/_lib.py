@@ -19,6 +19,7 @@ LIB_PATH = os.path.join(HERE, "libmoe.so")
 MOE_OK, MOE_ERR_INVALID_ARG, MOE_ERR_CUDA, MOE_ERR_DEVICE_CHECK, MOE_ERR_TIMEOUT, \
     MOE_ERR_UNSUPPORTED = range(6)
 MOE_F32, MOE_BF16 = 0, 1
+MOE_PAIRS_OFF, MOE_PAIRS_ALL, MOE_PAIRS_AUTO = 0, 1, 2
 
 
 class MoEError(RuntimeError):
@@ -77,6 +78,7 @@ _SIGS = {
     "moe_set_wait_limit_ns": [ctypes.c_uint64],
     "moe_set_gemm_pairs": [ctypes.c_int],
     "moe_mse_loss": [_CFG] + [P] * 5 + [ctypes.c_size_t, P],
+    "moe_expert_ffn_bwd_kernels": [_CFG, ctypes.POINTER(ctypes.c_int32)],
     "moe_sgd_update": [P, P, P, ctypes.c_int64, ctypes.c_int64, P, ctypes.c_float, ctypes.c_int, P],
 }
 for _n, _a in _SIGS.items():
@@ -200,6 +202,12 @@ def moe_expert_ffn_fwd(cfg, x_perm, offsets, w1, w2, h_gu, act, y_perm, x=None, 
                        stream=None):
     _call("moe_expert_ffn_fwd", cfg, x_perm, offsets, w1, w2, h_gu, act, y_perm, x, ws1, ws2,
           h_gu_sh, act_sh, y_sh, group_expert, stream=stream)
+
+
+def moe_expert_ffn_bwd_kernels(cfg) -> int:
+    n = ctypes.c_int32(0)
+    _check(_lib.moe_expert_ffn_bwd_kernels(ctypes.byref(cfg), ctypes.byref(n)), "moe_expert_ffn_bwd_kernels")
+    return int(n.value)
 
 
 def moe_mse_loss(cfg, out, target, loss, dout, workspace, workspace_bytes, stream=None):

@@ -1174,11 +1174,17 @@ void set_gemm_pairs(int mode) { tc::g_pairs = mode; }
 
 // Pair tiles where they fill at least four rounds of the SMs (the last, partly empty
 // round then costs little) and the operand feed, not the epilogue, bounds the tile.
+// The input-gradient GEMM (plain store, MN-major weights, a long contraction) takes
+// pairs with fewer tiles too: an SM ingests at most ~145 GB/s from L2 with TMA, which
+// caps a single-CTA 128 x 256 tile near 80% of the MMA rate and a pair's 256 x 256 tile
+// (half the B bytes per SM) does not, and its weight-gradient partner then runs beside
+// it on the second stream.
 bool gemm_m_uses_pairs(const GemmMArgs& g) {
     using namespace tc;
     if (g.N % 256 != 0) return false;
     if (g_pairs == MOE_PAIRS_ALL) return true;
     if (g_pairs != MOE_PAIRS_AUTO || g.epi == EPI_SWIGLU_BWD) return false;
+    if (g.epi == EPI_STORE && !g.b_kmajor && g.K >= 512) return true;
     const int64_t pt_ub = g.rows.offsets ? ((int64_t)g.rows.rows + 2 * BM - 1) / (2 * BM) + g.G
                                          : (int64_t)g.G * ((g.rows.rows + 2 * BM - 1) / (2 * BM));
     return pt_ub * (g.N / 256) >= 4 * (int64_t)(sm_count() / 2);

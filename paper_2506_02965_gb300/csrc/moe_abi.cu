@@ -538,7 +538,7 @@ moe_status moe_expert_ffn_bwd(const moe_config* cfg, const void* x_perm, const i
     // CTA-pair tiles, and the CUDA-core path, instead put the weight gradient on a side
     // stream: dW2 alongside dA, dW1 alongside dX once dH exists.
     const bool fuse_a = bf16 && !gemm_m_uses_pairs(a);
-    const bool fuse_b = bf16 && !gemm_m_uses_pairs(b);
+    const bool fuse_b = bf16 && !gemm_m_uses_pairs(b);  // the same rule as moe_expert_ffn_bwd_kernels
     SideStream* ss = nullptr;
     if (!fuse_a || !fuse_b) {
         if ((st = cuda_status(side_stream(&ss), "side stream"))) return st;
@@ -671,6 +671,33 @@ moe_status moe_dispatch_bwd(const moe_config* cfg, const void* dx_perm, const in
                                                cfg->T, cfg->d_model, cfg->top_k,
                                                cfg->dtype == MOE_BF16, dx, (cudaStream_t)stream),
                        "moe_dispatch_bwd");
+}
+
+moe_status moe_expert_ffn_bwd_kernels(const moe_config* cfg, int32_t* count) {
+    moe_status st = check_cfg(cfg);
+    if (st) return st;
+    REQUIRE(count);
+    const bool bf16 = cfg->dtype == MOE_BF16;
+    const int64_t TK = cfg->T * cfg->top_k;
+    static const int32_t marker = 0;  // offsets mode: only its non-null-ness is looked at
+    GemmMArgs a{}, b{};
+    a.G = b.G = cfg->n_experts;
+    a.rows = b.rows = GroupRows{&marker, (int)TK, 0, 0, 0};
+    a.b_kmajor = b.b_kmajor = false;
+    a.N = cfg->d_ff;
+    a.K = cfg->d_model;
+    a.epi = EPI_SWIGLU_BWD;
+    b.N = cfg->d_model;
+    b.K = 2 * cfg->d_ff;
+    b.epi = EPI_STORE;
+    int n = 0;
+    if (TK > 0) {
+        n += (bf16 && !gemm_m_uses_pairs(a)) ? 1 : 2;
+        n += (bf16 && !gemm_m_uses_pairs(b)) ? 1 : 2;
+    }
+    if (cfg->n_shared && cfg->T > 0) n += 4;
+    *count = n;
+    return MOE_OK;
 }
 
 moe_status moe_mse_loss(const moe_config* cfg, const void* out, const void* target, float* loss,

@@ -274,13 +274,13 @@ class MoELayer:
     def kernels_per_step(self) -> int:
         """CUDA kernels this library launches per step (memsets not counted):
         route 1, aux 1, dispatch 3, expert fwd 2, combine 1, combine bwd 1,
-        unpermute-reduce 1; expert bwd: bf16 2 (dA with dW2, dX with dW1; 4 when a
-        backward GEMM runs as CTA-pair tiles, large workloads), fp32 4;
-        router backward: bf16 5 (dlogits, chunk dbias, dW_r partial GEMM, reduce,
-        dx_router GEMM), fp32 4 (dlogits, partials, reduce, dx_router GEMM); shared
-        experts add 2 + 4."""
+        unpermute-reduce 1; the expert backward as moe_expert_ffn_bwd_kernels reports it
+        (its shared experts included); router backward: bf16 5 (dlogits, chunk dbias,
+        dW_r partial GEMM, reduce, dx_router GEMM), fp32 4 (dlogits, partials, reduce,
+        dx_router GEMM); shared experts add 2 to the forward."""
         bf16 = self.shape.dtype == "bf16"
-        return 10 + (2 if bf16 else 4) + (5 if bf16 else 4) + (6 if self.shape.n_shared else 0)
+        return (10 + L.moe_expert_ffn_bwd_kernels(self.cfg) + (5 if bf16 else 4)
+                + (2 if self.shape.n_shared else 0))
 
     def check_status(self, stream=None):
         code = L.moe_device_status(stream)
