@@ -308,8 +308,8 @@ moe_status moe_device_status(moe_stream_t stream, int32_t* code /* HOST out */);
  * (default 2e9). A wait that runs out records MOE_ERR_TIMEOUT and the kernel returns. */
 moe_status moe_set_wait_limit_ns(uint64_t ns);
 
-/* Tile shape of the 256-wide expert GEMMs whose rows vary per expert (forward, dA,
- * dX), for all later calls of this process. A CTA-pair tile is 256 x 256, computed by
+/* Tile shape of the 256-wide expert GEMMs (forward, dA, dX and the weight gradients),
+ * for all later calls of this process. A CTA-pair tile is 256 x 256, computed by
  * two CTAs on two SMs with tcgen05 cta_group::2 MMAs, each SM holding half of the B
  * operand (half the operand traffic per SM of a single-CTA 128 x 256 tile), but twice
  * as few tiles share the SMs, so a launch with few tiles loses to its last round.
@@ -319,6 +319,9 @@ moe_status moe_set_wait_limit_ns(uint64_t ns);
  *                   (contraction 2F) and wherever a launch has at least four rounds
  *                   of them, except under the SwiGLU backward epilogue (which, not the
  *                   operand feed, bounds the dA GEMM).
+ * The weight-gradient GEMMs launched on their own (dW1; dW2 when dA runs as pairs; the
+ * shared experts') follow the same mode with 256 x 256 output tiles where both output
+ * dimensions are multiples of 256.
  * Results agree up to fp32 summation order. Any other mode: MOE_ERR_INVALID_ARG. */
 enum { MOE_PAIRS_OFF = 0, MOE_PAIRS_ALL = 1, MOE_PAIRS_AUTO = 2 };
 moe_status moe_set_gemm_pairs(int mode);

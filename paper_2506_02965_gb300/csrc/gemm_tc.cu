@@ -160,6 +160,12 @@ __device__ __forceinline__ void mma_commit_pair(uint32_t bar, uint16_t mask) {
         "h"(mask)
         : "memory");
 }
+// credit `bytes` of expected transactions to a barrier in another CTA of the cluster, as
+// if that many bytes had arrived there (no arrival)
+__device__ __forceinline__ void mbar_complete_tx_remote(uint32_t cluster_bar, uint32_t bytes) {
+    asm volatile("mbarrier.complete_tx.relaxed.cluster.shared::cluster.b64 [%0], %1;" ::"r"(cluster_bar), "r"(bytes)
+                 : "memory");
+}
 __device__ __forceinline__ void cluster_sync_all() {
     asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::
                      : "memory");
@@ -431,7 +437,9 @@ __global__ void __launch_bounds__(THREADS, 1)
     constexpr int TMEM_COLS = (2 * BN <= 32) ? 32 : (2 * BN <= 64) ? 64 : (2 * BN <= 128) ? 128 : (2 * BN <= 256) ? 256 : 512;
 
     extern __shared__ uint8_t smem_raw[];
-    __shared__ uint64_t bars[2 * NST + 5 + 2 * EPI_WARPS];
+    // K-variable pairs: the peer's own barriers for the partial last k-block of a tile
+    constexpr int NPART = (PAIR && VAR_K) ? NST : 0;
+    __shared__ uint64_t bars[2 * NST + 5 + 2 * EPI_WARPS + NPART];
     __shared__ uint32_t s_tmem;
     __shared__ int s_abort;
     __shared__ int s_tile_start[MAX_GROUPS + 1];
@@ -557,6 +565,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     auto tfull_bar = [&](int a) { return bar0 + 8u * (2 * NST + a); };
     auto tempty_bar = [&](int a) { return bar0 + 8u * (2 * NST + 2 + a); };
     const uint32_t drain_bar = bar0 + 8u * (2 * NST + 4);
+    auto pfull_bar = [&](int s) { return bar0 + 8u * (2 * NST + 5 + 2 * EPI_WARPS + s); };
     // waits: cluster-scope acquire when the barrier also collects the peer's arrivals
     auto wait_bar = [&](uint32_t bar, uint32_t parity) -> bool {
         if constexpr (PAIR) {
@@ -587,6 +596,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
         mbar_init(drain_bar, 1);
         for (int i = 0; i < 2 * EPI_WARPS; ++i) mbar_init(bar0 + 8u * (2 * NST + 5 + i), 1);
+        for (int s = 0; s < NPART; ++s) mbar_init(pfull_bar(s), 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     if (warp == 1) {
@@ -621,10 +631,14 @@ __global__ void __launch_bounds__(THREADS, 1)
             uint32_t phase = 0;
             int issued_phase[NST];
             for (int s = 0; s < NST; ++s) issued_phase[s] = -1;
+            // K-variable pair peer: stages whose own barrier was ever armed, and per stage
+            // the parity of the next phase to arm
+            uint32_t parmed = 0, pnext = 0;
             bool ok = true;
             // every TMA load is counted on the leader's full barrier (CTA 0 of a pair)
+            bool local_bar = false;  // this stage's copies complete on this CTA's own barrier
             auto load = [&](uint32_t dst, const CUtensorMap* map, uint32_t fb, int c0, int c1) {
-                if constexpr (PAIR) tma_load_2d_pair(dst, map, fb, c0, c1);
+                if (PAIR && !local_bar) tma_load_2d_pair(dst, map, fb, c0, c1);
                 else tma_load_2d(dst, map, fb, c0, c1);
             };
             for (int t = tile0; t < total_tiles && ok; t += tile_step) {
@@ -636,7 +650,13 @@ __global__ void __launch_bounds__(THREADS, 1)
                     }
                     const uint32_t sa = ring + stage * STAGE_BYTES;
                     const uint32_t sb = sa + A_BYTES;
-                    const uint32_t fb = PAIR ? map_to_rank(full_bar(stage), 0) : full_bar(stage);
+                    // K-variable pair, peer, partial last k-block: its copies land on its own
+                    // barrier; the MMA warp zeroes the rows past the group's end and then
+                    // credits these bytes to the leader's full barrier
+                    const bool part_peer = PAIR && VAR_K && rank == 1 && kb == ti.k_iters - 1 && ti.last_rows < BK;
+                    const uint32_t fb = part_peer ? pfull_bar(stage)
+                                                  : (PAIR ? map_to_rank(full_bar(stage), 0) : full_bar(stage));
+                    local_bar = part_peer;
                     // In a pair only the leader arrives, expecting the bytes of both CTAs: the
                     // peer's copies complete on the leader's barrier without an arrival (a
                     // cluster-scope arrive per stage cost the producers most of their time). The
@@ -644,6 +664,11 @@ __global__ void __launch_bounds__(THREADS, 1)
                     // always count towards the phase the leader arms.
                     if constexpr (PAIR) {
                         if (rank == 0) mbar_expect_tx(full_bar(stage), NPAIR * STAGE_BYTES);
+                        else if (part_peer) {
+                            mbar_expect_tx(fb, STAGE_BYTES);
+                            parmed |= 1u << stage;
+                            pnext ^= 1u << stage;
+                        }
                     } else {
                         mbar_expect_tx(fb, STAGE_BYTES);
                     }
@@ -680,6 +705,18 @@ __global__ void __launch_bounds__(THREADS, 1)
                     if (++stage == NST) {
                         stage = 0;
                         phase ^= 1u;
+                    }
+                }
+            }
+            if constexpr (PAIR && VAR_K) {
+                if ((!ok || *abort_flag) && rank == 1) {
+                    // partial copies on this CTA's own barriers: the last phase armed
+                    for (int s2 = 0; s2 < NST; ++s2) {
+                        if (!((parmed >> s2) & 1u)) continue;
+                        const uint32_t par = ((pnext >> s2) & 1u) ^ 1u;
+                        const uint64_t t0 = gtimer();
+                        while (!mbar_try(pfull_bar(s2), par) && gtimer() - t0 < drain_limit) {
+                        }
                     }
                 }
             }
@@ -788,6 +825,47 @@ __global__ void __launch_bounds__(THREADS, 1)
             }
         }
         __syncwarp();
+        if constexpr (PAIR && VAR_K) {
+            // Peer of a K-variable pair: the leader's MMAs read this CTA's A rows too, so
+            // the rows of a tile's last k-block past its group's end are zeroed here, as
+            // the leader does for its own; then this stage's bytes are credited to the
+            // leader's full barrier, which the peer's copies did not count.
+            if (rank == 1) {
+                int st2 = 0;
+                uint32_t wpar = 0;  // per stage: parity of the next partial phase to wait for
+                bool ok2 = true;
+                for (int t = tile0; t < total_tiles && ok2; t += tile_step) {
+                    const Tile ti = tile_at(t);
+                    for (int kb = 0; kb < ti.k_iters; ++kb) {
+                        if (kb == ti.k_iters - 1 && ti.last_rows < BK) {
+                            if (!mbar_wait(pfull_bar(st2), (wpar >> st2) & 1u, abort_flag, p.wait_ns)) {
+                                ok2 = false;
+                                break;
+                            }
+                            wpar ^= 1u << st2;
+                            const int zr0 = ti.last_rows, zr1 = ((ti.last_rows + 15) / 16) * 16;
+                            if (zr1 > zr0) {
+                                uint8_t* base = ring_ptr + (size_t)st2 * STAGE_BYTES;
+                                const int per_box = (zr1 - zr0) * 8;  // 16-byte words
+#pragma unroll
+                                for (int b = 0; b < BM / 64; ++b) {
+                                    uint4* z = reinterpret_cast<uint4*>(base + b * 8192 + zr0 * 128);
+                                    for (int i = lane; i < per_box; i += 32) z[i] = make_uint4(0, 0, 0, 0);
+                                }
+                                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                            }
+                            __syncwarp();
+                            if (lane == 0) {
+                                asm volatile("fence.acq_rel.cluster;" ::: "memory");
+                                mbar_complete_tx_remote(map_to_rank(full_bar(st2), 0), STAGE_BYTES);
+                            }
+                            __syncwarp();
+                        }
+                        if (++st2 == NST) st2 = 0;
+                    }
+                }
+            }
+        }
     } else {
         // ------------------------------------------------------------ epilogue warps 2-5
         // Warp w reads TMEM lane quarter w % 4 (32 rows). Finished 32x32 bf16 boxes are
@@ -1190,6 +1268,17 @@ bool gemm_m_uses_pairs(const GemmMArgs& g) {
     return pt_ub * (g.N / 256) >= 4 * (int64_t)(sm_count() / 2);
 }
 
+// K-variable weight gradients (dW = A^T B over each group's rows) as 256 x 256 CTA-pair
+// tiles: both output dimensions multiples of 256, and (AUTO) at least four rounds of
+// pair tiles.
+bool gemm_k_uses_pairs(const GemmKArgs& g) {
+    using namespace tc;
+    if (g.epi != EPI_STORE || g.M % 256 != 0 || g.N % 256 != 0) return false;
+    if (g_pairs == MOE_PAIRS_ALL) return true;
+    if (g_pairs != MOE_PAIRS_AUTO) return false;
+    return (int64_t)g.G * (g.M / 256) * (g.N / 256) >= 4 * (int64_t)(sm_count() / 2);
+}
+
 // M-variable grouped GEMM (forward, dA, dX).
 cudaError_t launch_gemm_m(const GemmMArgs& g, bool bf16, cudaStream_t s) {
     if (!bf16) return launch_gemm_m_simt(g, s);
@@ -1298,6 +1387,8 @@ cudaError_t launch_gemm_k(const GemmKArgs& g, bool bf16, cudaStream_t s) {
         return launch<64, true, true, EPI_DWR>(ma, mb, ma, ma, p, tiles, s);
     }
     if (!make_map(&mo, g.out, g.N, (int64_t)g.G * g.M, 0, true)) return cudaErrorInvalidValue;
+    if (gemm_k_uses_pairs(g))
+        return launch<256, true, true, EPI_STORE, true>(ma, mb, mo, mo, p, (int64_t)g.G * (g.M / 256) * (g.N / 256), s);
     if (g.N % 256 == 0) return launch<256, true, true, EPI_STORE>(ma, mb, mo, mo, p, tiles * (g.N / 256), s);
     return launch<128, true, true, EPI_STORE>(ma, mb, mo, mo, p, tiles * (g.N / 128), s);
 }

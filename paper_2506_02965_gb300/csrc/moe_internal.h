@@ -139,6 +139,7 @@ cudaError_t launch_gemm_k(const GemmKArgs& g, bool bf16, cudaStream_t s);
 cudaError_t launch_gemm_mk(const GemmMArgs& m, const GemmKArgs& k, cudaStream_t s);
 // whether launch_gemm_m runs this GEMM as CTA-pair tiles (bf16)
 bool gemm_m_uses_pairs(const GemmMArgs& g);
+bool gemm_k_uses_pairs(const GemmKArgs& g);
 void set_wait_limit_ns(uint64_t ns);
 void set_gemm_pairs(int mode);  // MOE_PAIRS_*
 cudaError_t gemm_status(cudaStream_t s, int* code);
