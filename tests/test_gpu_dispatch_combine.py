@@ -32,7 +32,15 @@ def picks(T, E, k, pattern, seed=0):
         return np.asarray(out, np.int32)
     if pattern == "all":  # k == E
         return np.stack([rng.permutation(E) for _ in range(T)]).astype(np.int32)
+    if pattern == "edges":  # k == 1: expert sizes at the 16- and 64-row boundaries
+        sizes = np.array(EDGE_SIZES[:E])
+        assert k == 1 and sizes.sum() == T
+        return rng.permutation(np.repeat(np.arange(E), sizes)).astype(np.int32)[:, None]
     raise ValueError(pattern)
+
+
+# rows per expert around the K=16 MMA step and the 64-row k-block (empty, one row, ...)
+EDGE_SIZES = [0, 1, 15, 16, 17, 63, 64, 65, 128, 200]
 
 
 CASES = [(1000, 8, 2, "uniform", "bf16"), (333, 16, 2, "skewed", "bf16"),

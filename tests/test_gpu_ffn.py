@@ -120,14 +120,17 @@ def test_expert_ffn_is_deterministic(L):
 
 @pytest.mark.parametrize("pairs", [0, 1, 2])
 def test_expert_ffn_single_cta_and_pair_tiles(L, pairs):
-    """The 256-wide M-variable GEMMs in every tile mode: one CTA per 128x256 tile, a CTA
-    pair per 256x256 tile, or the automatic choice per launch (ragged experts, an empty
-    expert, a skewed split)."""
+    """The 256-wide GEMMs in every tile mode: one CTA per 128x256 tile, a CTA pair per
+    256x256 tile, or the automatic choice per launch (ragged experts, an empty expert, a
+    skewed split, experts ending at every offset of a k-block)."""
     L.moe_set_gemm_pairs(pairs)
     try:
         for case in [(777, 512, 8, 512, 2, "skewed", "bf16", 0, 0),
                      (300, 256, 4, 256, 2, "uniform", "bf16", 1, 256),
-                     (1024, 1024, 16, 2816, 2, "uniform", "bf16", 0, 0)]:
+                     (1024, 1024, 16, 2816, 2, "uniform", "bf16", 0, 0),
+                     # experts of 0, 1, 15, 16, 17, 63, 64, 65, 128, 200 rows: every way the
+                     # weight gradients' last k-block can end (pairs: zeroed on both CTAs)
+                     (569, 256, 10, 256, 1, "edges", "bf16", 0, 0)]:
             test_expert_ffn_fwd_bwd(L, case)
     finally:
         L.moe_set_gemm_pairs(2)
