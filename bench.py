@@ -4,8 +4,10 @@
 A step is one pass of the whole layer (gating, aux loss, dispatch, expert FFN
 forward, combine, combine backward, expert FFN backward, gating backward,
 unpermute-reduce) over one batch of seeded synthetic tokens. The default workload
-is mid_bf16 (T=4096, d=1024, E=16 SwiGLU experts of F=2816, top-2, bf16 storage
-with fp32 accumulation).
+is large_zipf_bf16, the largest layer that fits one GPU: T=16384 tokens, d=4096,
+E=8 SwiGLU experts of F=14336, top-2, router bias giving Zipf(1.2) expert
+popularity, bf16 storage with fp32 accumulation (34.6 TFLOP of expert GEMMs per
+step).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
   python bench.py --impl reference ...   # the fp64 CPU oracle on the host cores
@@ -16,7 +18,13 @@ every timed step. Under torchrun each rank runs its own replica (the layer does 
 shard; no collective on the data path); the time is the max over ranks and the
 value is the tokens of all ranks per second. Prints one JSON line on rank 0.
 
-e2e: the same layer fed from pinned host buffers through MoELayer.run_host, K passes
+Rooflines: a second pass runs the layer's calls one after another on one stream,
+each bracketed by its own events with L2 flushed before it, and reports every
+memory-bound stage's algorithmic bytes / its time against the measured HBM copy
+bandwidth, and the expert GEMM calls' algorithmic flops / their time against the
+measured bf16 tensor peak.
+
+e2e: the same layer fed from pinned host buffers through MoELayer.run_host, passes
 whose host->device uploads (x, dOut) and device->host downloads (out, dx, aux loss)
 are all inside one timed region, pipelined with the neighbouring passes' kernels.
 """
@@ -38,15 +46,17 @@ from synth import moe_inputs as mi  # noqa: E402
 
 METRIC = "MoE layer fwd+bwd tokens/s on 1 GB300"
 FLUSH_BYTES = 256 << 20
+# dense bf16 tensor-core rate of one GB300 as NVIDIA states it (without 2:4 sparsity)
+NOMINAL_BF16_TFLOPS = 2250.0
 
 
 def args_():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=300)
-    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--steps", type=int, default=60)
+    ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--workload", default="mid_bf16")
+    ap.add_argument("--workload", default="large_zipf_bf16")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
@@ -76,22 +86,35 @@ def workload_desc(sh):
 
 
 # --------------------------------------------------------------------------- memory bytes
-def mem_bytes_per_step(sh) -> float:
-    """Algorithmic HBM bytes of the memory-bound stages per step:
-    route read x + write logits/probs/picks; dispatch read x + write x_perm + tables;
-    combine read y_perm, w + write out; combine bwd read dout, y_perm + write dy, dw;
-    route bwd read probs, dw, x + write dlogits; unpermute read dx_perm (+ dlogits)
-    + write dx."""
+def stage_bytes(sh) -> dict:
+    """Algorithmic HBM bytes per step of each memory-bound call: what the layer must
+    read and write, per token (b = bytes per activation element), times T:
+      route (gating, a1-a3)      read x: d b;              write probs, picks: 4E + 8k
+      aux (load-balancing loss)  read probs: 4E
+      dispatch (a5-a8)           read x: d b;              write x_perm: k d b; tables: 12k
+      combine_fwd (a11)          read y_perm, w: k d b + 4k (+ S d b shared outputs); write out: d b
+      combine_bwd (a12)          read dout, y_perm: d b + k d b; write dy_perm, dw: k d b + 4k
+      route_bwd (a17)            read probs, dprobs, x, dx-side: 8E + 2 d b; write dx_router: d b
+      dispatch_bwd (a18)         read dx_perm: k d b (+ S d b shared dx); write dx: d b
+    Re-reads, padding and the weights of the router (P E d b, not per token) do not
+    count."""
     b = 2 if sh.dtype == "bf16" else 4
-    T, d, E, k = sh.T, sh.d_model, sh.n_experts, sh.top_k
-    per_tok = 0.0
-    per_tok += d * b + 2 * E * 4 + k * 8                     # route
-    per_tok += d * b + k * d * b + 12 * k                    # dispatch
-    per_tok += k * d * b + k * 4 + d * b                     # combine fwd
-    per_tok += d * b + k * d * b + k * d * b + k * 4         # combine bwd
-    per_tok += 2 * E * 4 + k * 4 + d * b + E * 4             # route bwd
-    per_tok += k * d * b + E * 4 + d * b                     # unpermute-reduce
-    return per_tok * T
+    T, d, E, k, S = sh.T, sh.d_model, sh.n_experts, sh.top_k, sh.n_shared
+    per = {
+        "route": d * b + 4 * E + 8 * k,
+        "aux": 4 * E,
+        "dispatch": d * b + k * d * b + 12 * k,
+        "combine_fwd": k * d * b + 4 * k + S * d * b + d * b,
+        "combine_bwd": d * b + k * d * b + k * d * b + 4 * k,
+        "route_bwd": 8 * E + 2 * d * b + d * b,
+        "dispatch_bwd": k * d * b + S * d * b + d * b,
+    }
+    return {n: v * T for n, v in per.items()}
+
+
+def mem_bytes_per_step(sh) -> float:
+    """Algorithmic HBM bytes of all memory-bound calls of one step (stage_bytes summed)."""
+    return float(sum(stage_bytes(sh).values()))
 
 
 # --------------------------------------------------------------------------- clocks
@@ -158,38 +181,84 @@ def gemm_traffic_record(sh):
 
 
 # --------------------------------------------------------------------------- oracle legs
-def oracle_sample(workload: str, tokens: int, repeats: int) -> dict:
-    """Time the fp64 oracle (fwd+bwd) on the first `tokens` tokens of the workload."""
-    import numpy as np
+# Both CPU legs (cpu_baseline in our arm's line, and the whole --impl reference arm)
+# time the fp64 oracle as it stands on the same sample and with the same policy: the
+# first `sample_tokens` tokens of the workload (all experts, fp64 forward + backward),
+# the mean over the timed repeats after untimed warm-up repeats. The sample size comes
+# from one probe pass so that K + W repeats of it take about REF_BUDGET_S seconds; it
+# depends only on the workload and K + W, so both legs of one driver round (the same
+# --steps and --warmup) time the same tokens.
+REF_BUDGET_S = 150.0
+CPU_BASELINE_S = 15.0  # our arm's cpu_baseline: repeats of that sample for about this long
 
-    from oracle import moe_oracle as mo
+
+def _oracle_inputs(workload: str):
+    import numpy as np
     sh = mi.shape_by_name(workload)
     inp = mi.make_inputs(sh)
-    sub = {k: (np.asarray(v, np.float64) if isinstance(v, np.ndarray) and v.dtype == np.float32
-               else v) for k, v in inp.items()}
-    sub["x"] = sub["x"][:tokens]
-    sub["dout"] = sub["dout"][:tokens]
+    full = {k: (np.asarray(v, np.float64) if isinstance(v, np.ndarray) and v.dtype == np.float32
+                else v) for k, v in inp.items()}
+    return sh, full
+
+
+def _oracle_step(sh, full, tokens: int) -> float:
+    """One fwd+bwd of the oracle on the first `tokens` tokens; returns seconds."""
+    import numpy as np
+    from oracle import moe_oracle as mo
     P = sh.n_parties
+    tokens = max(P, tokens - tokens % P)
+    sub = dict(full)
+    sub["x"] = full["x"][:tokens]
+    sub["dout"] = full["dout"][:tokens]
     sub["party_offsets"] = (np.arange(P + 1) * (tokens // P)).astype(np.int32)
-    s2 = sh.with_(T=tokens - tokens % P)
-    times = []
-    for _ in range(repeats):
-        t0 = time.perf_counter()
-        f = mo.layer_forward(sub, s2)
-        mo.layer_backward(sub, s2, f)
-        times.append(time.perf_counter() - t0)
-    return {"tokens": s2.T, "seconds": times}
+    s2 = sh.with_(T=tokens)
+    t0 = time.perf_counter()
+    f = mo.layer_forward(sub, s2)
+    mo.layer_backward(sub, s2, f)
+    return time.perf_counter() - t0
 
 
-def cpu_baseline(workload: str, tokens: int, repeats: int) -> dict:
-    """Run oracle_sample in a fresh interpreter with every host core for BLAS."""
+def oracle_timing(workload: str, steps: int, warmup: int, sample_steps: int,
+                  sample_warmup: int, repeats: int | None = None,
+                  budget_s: float | None = None) -> dict:
+    """Time the oracle: size the sample from (sample_steps + sample_warmup) within
+    REF_BUDGET_S, then run `warmup` untimed and `steps` timed repeats of it (or, with
+    budget_s, as many timed repeats as fit about budget_s seconds, at least 2)."""
+    sh, full = _oracle_inputs(workload)
+    P = sh.n_parties
+    probe_tok = max(P, 16 - 16 % P)
+    _oracle_step(sh, full, probe_tok)             # first touch of the weights
+    t_probe = _oracle_step(sh, full, probe_tok)
+    t_fixed = _oracle_step(sh, full, P)           # per-step cost that does not scale with T
+    per_tok = max(t_probe - t_fixed, 1e-9) / max(probe_tok - P, 1)
+    per_step = REF_BUDGET_S / max(1, sample_steps + sample_warmup)
+    tokens = int(min(sh.T, max(P, (per_step - t_fixed) / per_tok)))
+    tokens = max(P, tokens - tokens % P)
+    for _ in range(warmup):
+        _oracle_step(sh, full, tokens)
+    secs = []
+    if budget_s is not None:
+        t_end = time.perf_counter() + budget_s
+        while len(secs) < 2 or time.perf_counter() < t_end:
+            secs.append(_oracle_step(sh, full, tokens))
+    else:
+        for _ in range(steps):
+            secs.append(_oracle_step(sh, full, tokens))
+    return {"tokens": tokens, "seconds": secs, "warmup": warmup}
+
+
+def run_oracle_subprocess(workload: str, steps: int, warmup: int, sample_steps: int,
+                          sample_warmup: int, budget_s: float | None = None) -> dict:
+    """oracle_timing in a fresh interpreter with every host core for BLAS (the GPU
+    process may hold a CUDA context; the oracle needs none)."""
     cores = os.cpu_count() or 1
     env = dict(os.environ, OPENBLAS_NUM_THREADS=str(cores), OMP_NUM_THREADS=str(cores),
                MKL_NUM_THREADS=str(cores), CUDA_VISIBLE_DEVICES="")
     code = (f"import json,sys; sys.path.insert(0,{ROOT!r}); import bench; "
-            f"print(json.dumps(bench.oracle_sample({workload!r}, {tokens}, {repeats})))")
+            f"print(json.dumps(bench.oracle_timing({workload!r}, {steps}, {warmup}, "
+            f"{sample_steps}, {sample_warmup}, budget_s={budget_s!r})))")
     r = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True,
-                       timeout=900)
+                       timeout=1800)
     if r.returncode:
         raise RuntimeError(r.stderr[-2000:])
     res = json.loads(r.stdout.strip().splitlines()[-1])
@@ -197,19 +266,19 @@ def cpu_baseline(workload: str, tokens: int, repeats: int) -> dict:
     return res
 
 
+def sample_desc(sh, res) -> str:
+    return (f"first {res['tokens']} tokens of {sh.name} (all experts), fp64 fwd+bwd per repeat; "
+            f"mean of {len(res['seconds'])} timed repeats after {res['warmup']} untimed; "
+            f"sample sized so that --steps + --warmup repeats take ~{REF_BUDGET_S:.0f} s")
+
+
 def run_reference(a):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return
     sh = mi.shape_by_name(a.workload)
-    # per-step sample sized from one probe step so that the whole run stays ~3 minutes
-    probe = cpu_baseline(a.workload, 64, 1)
-    per_tok = probe["seconds"][0] / 64
-    budget = 180.0 / max(1, a.steps + a.warmup)
-    tokens = int(max(sh.n_parties, min(sh.T, budget / max(per_tok, 1e-9))))
-    res = cpu_baseline(a.workload, tokens, a.steps + a.warmup)
-    secs = res["seconds"][a.warmup:]
-    ms = 1e3 * statistics.mean(secs)
+    res = run_oracle_subprocess(a.workload, a.steps, a.warmup, a.steps, a.warmup)
+    ms = 1e3 * statistics.mean(res["seconds"])
     value = res["tokens"] / (ms / 1e3)
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
@@ -218,9 +287,7 @@ def run_reference(a):
         "data": "synthetic (seeded numpy PCG64)",
         "config": {"workload": workload_desc(sh), "sample_tokens": res["tokens"]},
         "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": res["cores"],
-                         "kind": "oracle",
-                         "sample": f"first {res['tokens']} tokens of {sh.name}, all experts, "
-                                   f"fp64 fwd+bwd per step"},
+                         "kind": "oracle", "sample": sample_desc(sh, res)},
         "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }
@@ -334,6 +401,8 @@ def main():
     inp = mi.make_inputs(sh)
     lay = MoELayer(sh)
     lay.load(inp)
+    for name in ("w1", "w2", "ws1", "ws2"):  # on the device now; x and dOut stay for e2e
+        inp.pop(name, None)
     flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device="cuda")
     stream = torch.cuda.current_stream()
 
@@ -364,26 +433,27 @@ def main():
     lay.check_status()
     ms = statistics.mean([e0.elapsed_time(e1) for e0, e1 in ev])
 
-    # roofline split: a second pass with events also at the expert-GEMM call boundaries
-    # (an event between two kernels stops the next one from being scheduled early, so
-    # this pass is not the headline)
-    Km = max(3, min(K, 100))
-    names = ["start", "ffn_fwd_begin", "ffn_fwd_end", "ffn_bwd_begin", "ffn_bwd_end", "end"]
-    evm = [{n: torch.cuda.Event(enable_timing=True) for n in names} for _ in range(Km)]
+    # rooflines: the layer's calls one after another on one stream, each bracketed by
+    # its own events with L2 flushed before it (not the headline: the step overlaps the
+    # aux loss and the router backward with the expert calls on a side stream)
+    Ks = max(3, min(K, 20))
+    names = [n for n, _ in lay.STAGES]
+    evs = [{n: (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+            for n in names} for _ in range(Ks)]
     barrier()
     torch.cuda.synchronize()
-    for i in range(Km):
-        flush.fill_(i & 0xFF)
-        e = evm[i]
-        e["start"].record(stream)
-        lay.step(mark=lambda n, e=e: e[n].record(stream))
-        e["end"].record(stream)
+    for i in range(Ks):
+        for j, n in enumerate(names):
+            flush.fill_((i + j) & 0xFF)
+            evs[i][n][0].record(stream)
+            getattr(lay, n)(stream)
+            evs[i][n][1].record(stream)
     torch.cuda.synchronize()
     lay.check_status()
-    ms_marked = statistics.mean([e["start"].elapsed_time(e["end"]) for e in evm])
-    gms = statistics.mean([e["ffn_fwd_begin"].elapsed_time(e["ffn_fwd_end"]) +
-                           e["ffn_bwd_begin"].elapsed_time(e["ffn_bwd_end"]) for e in evm])
-    ms, gms, ms_marked = max_over_ranks([ms, gms, ms_marked], world)
+    stage_ms = {n: statistics.mean([e[n][0].elapsed_time(e[n][1]) for e in evs]) for n in names}
+    red = max_over_ranks([ms] + [stage_ms[n] for n in names], world)
+    ms, stage_ms = red[0], dict(zip(names, red[1:]))
+    gms = stage_ms["ffn_fwd"] + stage_ms["ffn_bwd"]
     value = world * sh.T / (ms / 1e3)
 
     # e2e: host buffers in, host results out, through the same public calls. The passes
@@ -397,7 +467,7 @@ def main():
         hd = torch.from_numpy(inp["dout"]).to(lay.dt).pin_memory()
         outs = [(torch.empty_like(hx).pin_memory(), torch.empty_like(hx).pin_memory(),
                  torch.empty(sh.n_parties, dtype=torch.float32).pin_memory()) for _ in range(2)]
-        Ke = max(3, min(K, 100))
+        Ke = max(3, min(K, 40))
         batches = [(hx, hd) + outs[i % 2] for i in range(Ke)]
         lay.run_host(batches[:max(3, a.warmup)], stream=stream)  # warm-up of the pipelined path
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -430,16 +500,30 @@ def main():
     from paper_2506_02965_gb300 import _lib as L
     n_gemm = 2 + L.moe_expert_ffn_bwd_kernels(lay.cfg) + (2 if sh.n_shared else 0)
     traffic = gemm_traffic_record(sh)
+    fwd_flops, bwd_flops = gemm_flops / 3.0, 2.0 * gemm_flops / 3.0
     roofline = {"bound": "tensor", "kernel": "grouped_gemm_kernel (tcgen05, all expert GEMM launches)",
                 "achieved": achieved, "peak": pk["bf16_tflops"], "unit": "TFLOP/s",
                 "frac": achieved / pk["bf16_tflops"], "traffic": traffic,
+                "peak_source": f"{pk['source']} bf16 burst (torch.matmul 8192^3, best of 10)",
                 "peak_sustained": pk["bf16_tflops_sustained"],
                 "frac_sustained": (achieved / pk["bf16_tflops_sustained"]
                                    if pk["bf16_tflops_sustained"] else None),
+                "peak_nominal": NOMINAL_BF16_TFLOPS,
+                "frac_nominal": achieved / NOMINAL_BF16_TFLOPS,
+                "flops_per_step": gemm_flops, "ms_per_step": gms,
                 "launches_per_step": n_gemm,
-                "peak_source": f"{pk['source']} bf16 burst"}
-    mem_ms = ms_marked - gms  # both from the marked pass
-    mem_gbs = mem_bytes_per_step(sh) / (mem_ms / 1e3) / 1e9
+                "calls": {"ffn_fwd": {"ms": stage_ms["ffn_fwd"],
+                                      "tflops": fwd_flops / stage_ms["ffn_fwd"] / 1e9},
+                          "ffn_bwd": {"ms": stage_ms["ffn_bwd"],
+                                      "tflops": bwd_flops / stage_ms["ffn_bwd"] / 1e9}},
+                "timing": "CUDA events around moe_expert_ffn_fwd and moe_expert_ffn_bwd, "
+                          f"mean of {Ks} serial passes"}
+    sb = stage_bytes(sh)
+    mem_stages = {n: {"bytes": sb[n], "ms": stage_ms[n],
+                      "gbs": sb[n] / (stage_ms[n] / 1e3) / 1e9,
+                      "frac": sb[n] / (stage_ms[n] / 1e3) / 1e9 / pk["hbm_gbs"]} for n in sb}
+    mem_bytes = sum(sb.values())
+    mem_ms = sum(stage_ms[n] for n in sb)
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": K,
         "warmup": a.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
@@ -449,12 +533,15 @@ def main():
                    "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
                    "l2": "flushed (256 MiB write) before every timed step"},
         "roofline": roofline,
-        "roofline_mem": {"bound": "hbm", "stages": "route, dispatch, combine, their bwd",
-                         "achieved": mem_gbs, "peak": pk["hbm_gbs"], "unit": "GB/s",
-                         "frac": mem_gbs / pk["hbm_gbs"],
-                         "note": "algorithmic bytes / (step time - expert GEMM time)"},
-        "gemm_ms_per_step": gms,
-        "marked_ms_per_step": ms_marked,
+        "roofline_mem": {"bound": "hbm", "achieved": mem_bytes / (mem_ms / 1e3) / 1e9,
+                         "peak": pk["hbm_gbs"], "unit": "GB/s",
+                         "frac": mem_bytes / (mem_ms / 1e3) / 1e9 / pk["hbm_gbs"],
+                         "peak_source": f"{pk['source']} HBM copy bandwidth",
+                         "bytes_per_step": mem_bytes, "ms_per_step": mem_ms,
+                         "stages": mem_stages,
+                         "timing": "CUDA events around each memory-bound call, L2 flushed "
+                                   f"before each, mean of {Ks} serial passes"},
+        "serial_ms_per_step": sum(stage_ms.values()),
         "gpu_launches": K * lay.kernels_per_step(),
         "wall_s_timed": wall,
     }
@@ -464,12 +551,10 @@ def main():
         line["clocks"] = clk
     if world == 1 and not a.no_cpu_baseline:
         try:
-            cb = cpu_baseline(a.workload, min(1024, sh.T), 2)
-            v = cb["tokens"] / min(cb["seconds"])
+            cb = run_oracle_subprocess(a.workload, 0, 1, a.steps, a.warmup, budget_s=CPU_BASELINE_S)
+            v = cb["tokens"] / statistics.mean(cb["seconds"])
             line["cpu_baseline"] = {"value": v, "unit": "tokens/s", "cores": cb["cores"],
-                                    "kind": "oracle",
-                                    "sample": f"first {cb['tokens']} tokens of {sh.name}, all "
-                                              f"experts, fp64 fwd+bwd, best of 2"}
+                                    "kind": "oracle", "sample": sample_desc(sh, cb)}
         except Exception as ex:  # reported, not fatal
             line["cpu_baseline"] = {"error": str(ex)[-300:]}
     print(json.dumps(line), flush=True)

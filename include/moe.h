@@ -157,8 +157,10 @@ moe_status moe_dispatch_owner(const moe_config* cfg, const int32_t* topk_idx, co
  *    It bounds the size: ceil(T/128) * E <= 65536 (e.g. T <= 131072 with E = 64);
  *    larger requests return MOE_ERR_INVALID_ARG and queue no work.
  *  - Calls no cudaMalloc or cudaFree. The first call on a device looks up the
- *    array's device address once (cudaGetSymbolAddress); make that first call before
- *    any stream capture.
+ *    array's device address once (cudaGetSymbolAddress) and keeps it for the process;
+ *    make that first call before any stream capture. The kept address belongs to the
+ *    device's context at that time: after cudaDeviceReset on that device, do not call
+ *    moe_dispatch_noalloc there again in this process.
  *  - Every call shares the one array. Each call overwrites the entries it uses, so
  *    back-to-back calls on one stream are fine; calls whose kernels overlap on the GPU
  *    (several streams or host threads at once) race and give wrong tables.
@@ -223,6 +225,10 @@ moe_status moe_combine_bwd(const moe_config* cfg, const void* dout, const void* 
  *   h_gu_sh, act_sh (forward), dh_sh [S,T,2Fs] out, dx_sh [S,T,d] out,
  *   dws1 [S,2Fs,d] out, dws2 [S,d,Fs] out.
  * group_expert: as in moe_expert_ffn_fwd (dw1[e], dw2[e] are always expert e's).
+ * Several host threads may call this at once: a weight gradient that runs on the
+ * library's second stream of the device (CTA-pair tiles, or fp32) is forked from and
+ * joined back to the caller's stream under a lock, so each call waits on its own
+ * stream's work only (calls on different streams then share that second stream).
  */
 moe_status moe_expert_ffn_bwd(const moe_config* cfg, const void* x_perm, const int32_t* offsets,
                               const void* w1, const void* w2, const void* h_gu, const void* act,

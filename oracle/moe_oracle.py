@@ -418,6 +418,55 @@ def layer_backward(inp: dict, shape, fwd: dict, dout=None, with_aux: bool = True
                 shared_grads=shared_grads, dx_router=dx_router)
 
 
+def router_backward(inp: dict, shape, probs, idx, topk_w, dtopk_w, aux_coef=None) -> dict:
+    """Backward of the gating function alone (Alg. 7; the router is trained as part of
+    the party's local layers, Sec. 3.1) for given picks I, gate weights w and their
+    gradients dw, with the picks held constant (R3):
+
+      dp_te = sum_j [I_tj = e] g_tj + dL_aux/dp_te,
+              g_tj = dw_tj, or (dw_tj - <dw_t, w_t>) / sum_j p_{t,I_tj} when renormalised;
+      dz_t  = p_t * (dp_t - <dp_t, p_t>)                  (softmax backward)
+      dW_r[q] = sum_{t in q} dz_t^T x_t;  db[q] = sum_{t in q} dz_t;  dx_router,t = dz_t W_r[q(t)]
+
+    The same steps as the router part of layer_backward, written for any picks: it needs
+    no expert output, so it runs at every workload size.
+    """
+    T, E, k = shape.T, shape.n_experts, shape.top_k
+    p = np.asarray(probs, f64)
+    idx = np.asarray(idx)
+    w = np.asarray(topk_w, f64)
+    dw = np.asarray(dtopk_w, f64)
+    dp = np.zeros((T, E), f64)
+    if shape.normalize_topk:
+        psel = np.take_along_axis(p, idx.astype(np.int64), axis=1)
+        S = psel.sum(axis=1)
+        inner = (dw * w).sum(axis=1)
+        for t in range(T):
+            for j in range(k):
+                dp[t, idx[t, j]] += (dw[t, j] - inner[t]) / S[t]
+    else:
+        for t in range(T):
+            for j in range(k):
+                dp[t, idx[t, j]] += dw[t, j]
+    po = np.asarray(inp["party_offsets"], dtype=np.int64)
+    part = party_of_tokens(T, po)
+    if aux_coef is not None:
+        dp += np.asarray(aux_coef, f64)[part]
+    dz = p * (dp - np.sum(dp * p, axis=1, keepdims=True))
+    x = np.asarray(inp["x"], f64)
+    Wr = np.asarray(inp["w_router"], f64)
+    P = Wr.shape[0]
+    dw_router = np.zeros_like(Wr)
+    dbias = np.zeros((P, E), f64)
+    dx_router = np.zeros((T, shape.d_model), f64)
+    for q in range(P):
+        rows = slice(po[q], po[q + 1])
+        dw_router[q] = dz[rows].T @ x[rows]
+        dbias[q] = dz[rows].sum(axis=0)
+        dx_router[rows] = dz[rows] @ Wr[q]
+    return dict(dprobs=dp, dlogits=dz, dw_router=dw_router, dbias=dbias, dx_router=dx_router)
+
+
 # ----------------------------------------------------------------------------- sampled
 
 def route_all(inp: dict, shape) -> dict:

@@ -63,7 +63,7 @@ def build(verbose: bool = False, extra: list[str] | None = None) -> str:
                 raise RuntimeError(f"nvcc failed on {cmd[-3]}")
     objs = [os.path.join(BUILD, s.replace(".cu", ".o")) for s in SOURCES]
     if jobs or not os.path.exists(LIB):
-        cmd = [cc, *ARCH, "-shared", "-o", LIB, *objs, "-lcudart_static" if False else "-cudart=static"]
+        cmd = [cc, *ARCH, "-shared", "-o", LIB, *objs, "-cudart=static"]
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode:
             sys.stderr.write(r.stdout + r.stderr)

@@ -3,13 +3,14 @@
 // Sec. 3.2). All memory-bound: 16-byte vector loads/stores, one warp per token or
 // per permuted row, no floating-point atomics (every result is deterministic).
 #include <algorithm>
+#include <atomic>
 
 #include "moe_common.cuh"
 #include "moe_internal.h"
 
 namespace moe {
 
-constexpr int DCH = 128;  // tokens per dispatch chunk (one thread each)
+constexpr int DCH = kDispatchChunkTokens;  // tokens per dispatch chunk (one thread each)
 
 // Per chunk: how many of its (token, pick) pairs went to each expert. Also checks
 // that every index lies in [0, E) and that no token picks an expert twice. With `send`
@@ -475,7 +476,10 @@ static __device__ __align__(256) int32_t g_dispatch_scratch[kNoAllocScratchInts]
 
 namespace {
 constexpr int kMaxDevices = 64;
-int32_t* g_scratch_ptr[kMaxDevices] = {};
+// Device address of g_dispatch_scratch per device, looked up on the first call there.
+// Two threads that make their first call at once both look it up and store the same
+// value; the atomic makes that well defined.
+std::atomic<int32_t*> g_scratch_ptr[kMaxDevices] = {};
 }  // namespace
 
 int64_t dispatch_noalloc_max_chunk_entries() { return kNoAllocScratchInts; }
@@ -487,13 +491,14 @@ cudaError_t launch_dispatch_noalloc(const int32_t* topk_idx, const void* x, int6
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
-    if (!g_scratch_ptr[dev]) {  // first call on this device: look the array up once
+    int32_t* cc = g_scratch_ptr[dev].load(std::memory_order_acquire);
+    if (!cc) {  // first call on this device: look the array up once
         void* p = nullptr;
         e = cudaGetSymbolAddress(&p, g_dispatch_scratch);
         if (e != cudaSuccess) return e;
-        g_scratch_ptr[dev] = static_cast<int32_t*>(p);
+        cc = static_cast<int32_t*>(p);
+        g_scratch_ptr[dev].store(cc, std::memory_order_release);
     }
-    int32_t* cc = g_scratch_ptr[dev];
     const int nch = (int)((T + DCH - 1) / DCH);
     if ((int64_t)nch * E > kNoAllocScratchInts) return cudaErrorInvalidValue;
     if (T == 0) return cudaMemsetAsync(offsets, 0, sizeof(int32_t) * (E + 1), s);

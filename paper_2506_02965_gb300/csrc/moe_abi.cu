@@ -90,7 +90,10 @@ size_t elem_size(const moe_config* c) { return c->dtype == MOE_BF16 ? 2 : 4; }
 // while the input-gradient GEMMs run on the caller's stream, so that the tail wave of
 // one persistent kernel is filled by the other. Fork and join are event waits, so all
 // work stays ordered with respect to the caller's stream. Created on the first call
-// on a device (that call must not be inside a stream capture).
+// on a device (that call must not be inside a stream capture). The events are shared
+// by every call on the device, so a call holds g_side_mu (side_stream's caller passes
+// its lock) from the fork record until its join wait is queued: two host threads
+// cannot re-record each other's events in between.
 struct SideStream {
     cudaStream_t s = nullptr;
     cudaEvent_t fork = nullptr, mid = nullptr, join = nullptr;
@@ -99,12 +102,12 @@ constexpr int kMaxDev = 64;
 SideStream g_side[kMaxDev];
 std::mutex g_side_mu;
 
+// Requires g_side_mu held by the caller.
 cudaError_t side_stream(SideStream** out) {
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     if (dev < 0 || dev >= kMaxDev) return cudaErrorInvalidDevice;
-    std::lock_guard<std::mutex> lk(g_side_mu);
     SideStream& ss = g_side[dev];
     if (!ss.s) {
         if ((e = cudaStreamCreateWithFlags(&ss.s, cudaStreamNonBlocking)) != cudaSuccess) return e;
@@ -301,7 +304,7 @@ moe_status moe_dispatch_noalloc(const moe_config* cfg, const int32_t* topk_idx, 
     moe_status st = check_cfg(cfg);
     if (st) return st;
     REQUIRE(offsets);
-    const int64_t nch = (cfg->T + 127) / 128;
+    const int64_t nch = (cfg->T + kDispatchChunkTokens - 1) / kDispatchChunkTokens;
     if (nch * cfg->n_experts > dispatch_noalloc_max_chunk_entries())
         return fail(MOE_ERR_INVALID_ARG,
                     "moe_dispatch_noalloc: ceil(T/128)*E = %lld exceeds its fixed scratch of %lld "
@@ -540,7 +543,9 @@ moe_status moe_expert_ffn_bwd(const moe_config* cfg, const void* x_perm, const i
     const bool fuse_a = bf16 && !gemm_m_uses_pairs(a);
     const bool fuse_b = bf16 && !gemm_m_uses_pairs(b);  // the same rule as moe_expert_ffn_bwd_kernels
     SideStream* ss = nullptr;
+    std::unique_lock<std::mutex> side_lock(g_side_mu, std::defer_lock);
     if (!fuse_a || !fuse_b) {
+        side_lock.lock();  // held until the join wait is queued (the events are shared)
         if ((st = cuda_status(side_stream(&ss), "side stream"))) return st;
         if ((st = cuda_status(cudaEventRecord(ss->fork, s), "fork"))) return st;
         if ((st = cuda_status(cudaStreamWaitEvent(ss->s, ss->fork, 0), "fork"))) return st;
@@ -562,6 +567,7 @@ moe_status moe_expert_ffn_bwd(const moe_config* cfg, const void* x_perm, const i
     if (ss) {
         if ((st = cuda_status(cudaEventRecord(ss->join, ss->s), "join"))) return st;
         if ((st = cuda_status(cudaStreamWaitEvent(s, ss->join, 0), "join"))) return st;
+        side_lock.unlock();
     }
     if (S) {
         GemmMArgs sa = a;

@@ -52,6 +52,7 @@ cudaError_t launch_route_bwd(const RouteBwdArgs& a, bool bf16, void* ws, cudaStr
 cudaError_t route_status(cudaStream_t s, int* code);
 
 // dispatch / combine
+constexpr int kDispatchChunkTokens = 128;  // tokens per dispatch chunk (per-chunk expert counts)
 size_t dispatch_workspace(int64_t T, int E);
 cudaError_t launch_dispatch(const int32_t* topk_idx, const void* x, int64_t T, int d, int E, int k,
                             bool bf16, int32_t* offsets, int32_t* slot_of, int32_t* token_of,

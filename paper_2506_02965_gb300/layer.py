@@ -108,63 +108,100 @@ class MoELayer:
     def _po(self):
         return self.party_offsets if self.shape.n_parties > 1 else None
 
+    # ------------------------------------------------------------------ stages
+    # One method per C-ABI call of the layer, each on the stream it is given. forward()
+    # and backward() chain them with the aux loss and the router backward on the side
+    # stream; a caller may also run them one by one on one stream (bench.py times each
+    # memory-bound stage that way).
+    def route(self, s):
+        L.moe_route(self.cfg, self.x, self.w_router, self.router_bias, self._po(), self.logits,
+                    self.probs, self.topk_idx, self.topk_w, self.counts, stream=s)
+
+    def aux(self, s):
+        L.moe_aux_loss(self.cfg, self.probs, self.counts, self._po(), self.aux_loss,
+                       self.aux_coef, stream=s)
+
+    def dispatch(self, s):
+        if self.owner_grouped:
+            L.moe_dispatch_owner(self.cfg, self.topk_idx, self.x, self.party_offsets,
+                                 self.group_expert, self.offsets, self.slot_of, self.token_of,
+                                 self.x_perm, self.send_counts, self.workspace, self.ws_bytes,
+                                 stream=s)
+        else:
+            L.moe_dispatch(self.cfg, self.topk_idx, self.x, self.offsets, self.slot_of,
+                           self.token_of, self.x_perm, self.workspace, self.ws_bytes, stream=s)
+
+    def ffn_fwd(self, s):
+        L.moe_expert_ffn_fwd(self.cfg, self.x_perm, self.offsets, self.w1, self.w2, self.h_gu,
+                             self.act, self.y_perm, self.x, self.ws1, self.ws2, self.h_gu_sh,
+                             self.act_sh, self.y_sh, group_expert=self.group_expert, stream=s)
+
+    def combine_fwd(self, s):
+        L.moe_combine_fwd(self.cfg, self.y_perm, self.topk_w, self.slot_of, self.y_sh, self.out,
+                          stream=s)
+
+    def combine_bwd(self, s):
+        L.moe_combine_bwd(self.cfg, self.dout, self.y_perm, self.topk_w, self.slot_of,
+                          self.dy_perm, self.dtopk_w, stream=s)
+
+    def route_bwd(self, s, with_aux: bool = True):
+        L.moe_route_bwd(self.cfg, self.x, self.w_router, self.probs, self.topk_idx, self.topk_w,
+                        self.dtopk_w, self.aux_coef if with_aux else None, self._po(),
+                        self.dlogits, self.dw_router, self.dbias, self.dx_router, self.workspace,
+                        self.ws_bytes, stream=s)
+
+    def ffn_bwd(self, s):
+        L.moe_expert_ffn_bwd(self.cfg, self.x_perm, self.offsets, self.w1, self.w2, self.h_gu,
+                             self.act, self.dy_perm, self.dh, self.dx_perm, self.dw1, self.dw2,
+                             self.x, self.dout, self.ws1, self.ws2, self.h_gu_sh, self.act_sh,
+                             self.dh_sh, self.dx_sh, self.dws1, self.dws2,
+                             group_expert=self.group_expert, stream=s)
+
+    def dispatch_bwd(self, s):
+        L.moe_dispatch_bwd(self.cfg, self.dx_perm, self.slot_of, self.dx_router, self.dx_sh,
+                           self.dx, stream=s)
+
+    # the calls of one step in order, with whether each is memory-bound (the expert FFN
+    # calls are the tensor-core GEMMs)
+    STAGES = (("route", True), ("aux", True), ("dispatch", True), ("ffn_fwd", False),
+              ("combine_fwd", True), ("combine_bwd", True), ("route_bwd", True),
+              ("ffn_bwd", False), ("dispatch_bwd", True))
+
     # ------------------------------------------------------------------ passes
     def forward(self, stream=None, mark=None):
-        c = self.cfg
         mark = mark or (lambda name: None)
         main = stream if stream is not None else torch.cuda.current_stream()
-        L.moe_route(c, self.x, self.w_router, self.router_bias, self._po(), self.logits,
-                    self.probs, self.topk_idx, self.topk_w, self.counts, stream=main)
+        self.route(main)
         # the aux loss needs only probs and counts: compute it beside the experts
         fork = torch.cuda.Event()
         fork.record(main)
         self.side.wait_event(fork)
-        L.moe_aux_loss(c, self.probs, self.counts, self._po(), self.aux_loss, self.aux_coef,
-                       stream=self.side)
+        self.aux(self.side)
         aux_done = torch.cuda.Event()
         aux_done.record(self.side)
-        if self.owner_grouped:
-            L.moe_dispatch_owner(c, self.topk_idx, self.x, self.party_offsets, self.group_expert,
-                                 self.offsets, self.slot_of, self.token_of, self.x_perm,
-                                 self.send_counts, self.workspace, self.ws_bytes, stream=main)
-        else:
-            L.moe_dispatch(c, self.topk_idx, self.x, self.offsets, self.slot_of, self.token_of,
-                           self.x_perm, self.workspace, self.ws_bytes, stream=main)
+        self.dispatch(main)
         mark("ffn_fwd_begin")
-        L.moe_expert_ffn_fwd(c, self.x_perm, self.offsets, self.w1, self.w2, self.h_gu, self.act,
-                             self.y_perm, self.x, self.ws1, self.ws2, self.h_gu_sh, self.act_sh,
-                             self.y_sh, group_expert=self.group_expert, stream=main)
+        self.ffn_fwd(main)
         mark("ffn_fwd_end")
-        L.moe_combine_fwd(c, self.y_perm, self.topk_w, self.slot_of, self.y_sh, self.out,
-                          stream=main)
+        self.combine_fwd(main)
         main.wait_event(aux_done)
 
     def backward(self, stream=None, with_aux: bool = True, mark=None):
-        c = self.cfg
         mark = mark or (lambda name: None)
         main = stream if stream is not None else torch.cuda.current_stream()
-        L.moe_combine_bwd(c, self.dout, self.y_perm, self.topk_w, self.slot_of, self.dy_perm,
-                          self.dtopk_w, stream=main)
+        self.combine_bwd(main)
         # the router backward needs only the gate gradients: run it beside the experts
         fork = torch.cuda.Event()
         fork.record(main)
         self.side.wait_event(fork)
-        L.moe_route_bwd(c, self.x, self.w_router, self.probs, self.topk_idx, self.topk_w,
-                        self.dtopk_w, self.aux_coef if with_aux else None, self._po(),
-                        self.dlogits, self.dw_router, self.dbias, self.dx_router, self.workspace,
-                        self.ws_bytes, stream=self.side)
+        self.route_bwd(self.side, with_aux)
         join = torch.cuda.Event()
         join.record(self.side)
         mark("ffn_bwd_begin")
-        L.moe_expert_ffn_bwd(c, self.x_perm, self.offsets, self.w1, self.w2, self.h_gu, self.act,
-                             self.dy_perm, self.dh, self.dx_perm, self.dw1, self.dw2, self.x,
-                             self.dout, self.ws1, self.ws2, self.h_gu_sh, self.act_sh, self.dh_sh,
-                             self.dx_sh, self.dws1, self.dws2, group_expert=self.group_expert,
-                             stream=main)
+        self.ffn_bwd(main)
         mark("ffn_bwd_end")
         main.wait_event(join)
-        L.moe_dispatch_bwd(c, self.dx_perm, self.slot_of, self.dx_router, self.dx_sh, self.dx,
-                           stream=main)
+        self.dispatch_bwd(main)
 
     def step(self, stream=None, mark=None):
         """One fwd+bwd pass of the whole layer. ``mark(name)`` (optional) is called at

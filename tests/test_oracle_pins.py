@@ -277,6 +277,52 @@ def test_gate_and_logit_gradients_finite_differences():
             assert abs((vals[0] - vals[1]) / (2 * h) - bwd["dlogits"][t, e]) < 1e-7
 
 
+@pytest.mark.parametrize("normalize", [0, 1])
+def test_router_backward_finite_differences(normalize):
+    """router_backward (the gating backward for given picks and gate gradients) is the
+    gradient of f = sum_tj c_tj w_tj + sum_te a_{p(t),e} p_te with the picks held fixed,
+    w and p as Alg. 7 defines them from z = W_r[p] x + b; checked by central differences
+    in W_r, b and x, and it agrees with the router part of the full layer backward."""
+    sh = tiny_shape(T=8, n_experts=5, top_k=2, normalize_topk=normalize, n_shared=0)
+    inp = tiny_inputs(sh, seed=31 + normalize)
+    rng = np.random.default_rng(5)
+    route = mo.route_all(inp, sh)
+    idx = route["topk_idx"]
+    c = rng.standard_normal((sh.T, sh.top_k))   # stands in for dL/dw
+    a = rng.standard_normal((sh.n_parties, sh.n_experts))  # stands in for dL_aux/dp
+    part = mo.party_of_tokens(sh.T, inp["party_offsets"])
+    rb = mo.router_backward(inp, sh, route["probs"], idx, route["topk_w"], c, a)
+
+    def f():
+        z = mo.router_logits(inp["x"], inp["w_router"], inp["router_bias"], inp["party_offsets"])
+        assert (mo.topk_indices(z.astype(np.float32), sh.top_k) == idx).all()
+        p = mo.softmax(z)
+        w = mo.gate_weights(p, idx, sh.normalize_topk)
+        return float(np.sum(c * w) + np.sum(a[part] * p))
+
+    h = 1e-6
+    for name, g in (("w_router", rb["dw_router"]), ("router_bias", rb["dbias"]),
+                    ("x", rb["dx_router"])):
+        base = inp[name]
+        for fi in range(base.size):
+            ii = np.unravel_index(fi, base.shape)
+            orig = base[ii]
+            base[ii] = orig + h
+            lp = f()
+            base[ii] = orig - h
+            lm = f()
+            base[ii] = orig
+            num = (lp - lm) / (2 * h)
+            assert abs(num - g[ii]) <= 1e-6 * max(1.0, abs(num)), (name, ii, num, g[ii])
+    # the same numbers as the router part of the whole layer's backward
+    fwd = mo.layer_forward(inp, sh)
+    bwd = mo.layer_backward(inp, sh, fwd)
+    rb2 = mo.router_backward(inp, sh, fwd["probs"], fwd["topk_idx"], fwd["topk_w"],
+                             bwd["dtopk_w"], fwd["aux_coef"])
+    for n in ("dlogits", "dw_router", "dbias", "dx_router"):
+        assert np.allclose(rb2[n], bwd[n], atol=1e-13, rtol=1e-12), n
+
+
 def test_layer_matches_independent_torch_autograd():
     """An independently written torch fp64 layer differentiated by autograd."""
     torch = pytest.importorskip("torch")

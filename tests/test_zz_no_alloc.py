@@ -6,11 +6,13 @@ workspace moe_dispatch needs. moe_dispatch_noalloc keeps that scratch in a fixed
 array inside the library. These tests call it through the C ABI and check that its
 tables and permuted rows equal those of moe_dispatch on the same inputs, exactly
 (integer and copy work), on two calls in a row, and that sizes beyond its fixed
-scratch are refused on the host.
+scratch are refused on the host. The tables are also checked directly against the
+oracle's dispatch tables (counting, prefix sums and stable slots written out on the CPU).
 """
 import numpy as np
 import pytest
 
+from oracle import moe_oracle as mo
 from synth import moe_inputs as mi
 from tests.gpu_util import cfg_of, dev, empty, need_gpu, status
 
@@ -27,8 +29,10 @@ def _both(L, T, d, E, k, dtype, seed):
     sh = mi.MoEShape("na", T, d, E, 128, k, dtype)
     cfg = cfg_of(L, sh)
     dt = torch.bfloat16 if dtype == "bf16" else torch.float32
-    idx = dev(_picks(T, E, k, seed), torch.int32)
-    x = dev(np.random.default_rng(seed + 1).standard_normal((T, d)).astype(np.float32), dt)
+    picks = _picks(T, E, k, seed)
+    xs = np.random.default_rng(seed + 1).standard_normal((T, d)).astype(np.float32)
+    idx = dev(picks, torch.int32)
+    x = dev(xs, dt)
     ws = L.moe_workspace_size(cfg)
     wsb = torch.empty(ws, dtype=torch.uint8, device="cuda")
     out = []
@@ -41,7 +45,7 @@ def _both(L, T, d, E, k, dtype, seed):
             L.moe_dispatch_noalloc(cfg, idx, x, *tabs)
         out.append(tabs)
     assert status(L) == 0
-    return out
+    return out, picks, x
 
 
 @pytest.mark.parametrize("T,d,E,k,dtype", [(4096, 1024, 16, 2, "bf16"), (1000, 256, 64, 6, "f32")])
@@ -49,9 +53,14 @@ def test_noalloc_dispatch_matches_workspace_dispatch_twice(T, d, E, k, dtype):
     import torch
     L = need_gpu()
     for call, seed in enumerate((11, 12)):  # two calls in a row share the fixed scratch
-        ref, got = _both(L, T, d, E, k, dtype, seed)
+        (ref, got), picks, x = _both(L, T, d, E, k, dtype, seed)
         for name, a, b in zip(("offsets", "slot_of", "token_of", "x_perm"), ref, got):
             assert torch.equal(a, b), (call, name)
+        _, off, slot, tok = mo.dispatch_tables(picks, E)
+        assert (got[0].cpu().numpy() == off).all(), call
+        assert (got[1].cpu().numpy() == slot.ravel()).all(), call
+        assert (got[2].cpu().numpy() == tok).all(), call
+        assert torch.equal(got[3], x[torch.as_tensor(tok, device="cuda")]), call
 
 
 def test_noalloc_dispatch_refuses_sizes_beyond_its_scratch():
