@@ -6,7 +6,11 @@ tolerance of the storage dtype):
   elementwise:  |gpu - ref| <= atol + rtol |ref| for every element, atol = rtol RMS(ref)
 The norm-wise bound reads "max relative error" per tensor; the elementwise one also
 catches an error confined to the small-magnitude rows or columns of a tensor, which
-the norm-wise bound would let through.
+the norm-wise bound would let through. A stack of independent tensors (one weight
+gradient per expert, one router gradient per party) is compared slice by slice
+(assert_close_slices): each slice's own scale sets its bounds, so neither a small
+expert's error hides under a large expert's max nor a large expert's rounding is
+held to a small expert's RMS.
 """
 import numpy as np
 
@@ -65,6 +69,18 @@ def assert_close(name, gpu, ref, tol):
     assert q <= 1.0, (f"{name}: elementwise |gpu-ref| exceeds {tol:.1e} (RMS(ref) + |ref|) "
                       f"by a factor {q:.2f}")
     return Err(e, q)
+
+
+def assert_close_slices(name, gpu, ref, tol):
+    """assert_close on every slice along the first axis; returns the worst slice's Err.
+    A slice whose reference is all zero (an expert no token picked) must be exactly
+    zero."""
+    ref = np.asarray(ref, np.float64)
+    worst = Err(0.0, 0.0)
+    for i in range(ref.shape[0]):
+        e = assert_close(f"{name}[{i}]", gpu[i], ref[i], tol)
+        worst = Err(max(float(e), float(worst)), max(e.elem, worst.elem))
+    return worst
 
 
 def ints(t):

@@ -8,7 +8,7 @@ import torch
 
 from oracle import moe_oracle as mo
 from synth import moe_inputs as mi
-from tests._cmp import TOL, assert_close
+from tests._cmp import TOL, assert_close, assert_close_slices
 from tests.gpu_util import cfg_of, dev, empty, need_gpu, status
 from tests.test_gpu_dispatch_combine import picks
 
@@ -78,8 +78,8 @@ def test_expert_ffn_fwd_bwd(L, case):
         ref["act"][r], ref["y"][r] = A, Y
         dH, dX, dW1, dW2 = mo.swiglu_backward(xp[r], w1[e], w2[e], G, U, A, dy[r].astype(np.float64))
         ref["dh"][r], ref["dxp"][r], ref["dw1"][e], ref["dw2"][e] = dH, dX, dW1, dW2
-    for n in ref:
-        assert_close(n, g[n], ref[n], tol)
+    for n in ref:  # weight gradients expert by expert
+        (assert_close_slices if n in ("dw1", "dw2") else assert_close)(n, g[n], ref[n], tol)
     if pattern == "skewed":  # the last expert got no rows: exact zero weight gradients
         assert off[E] - off[E - 1] == 0
         assert (g["dw1"][E - 1] == 0).all() and (g["dw2"][E - 1] == 0).all()
