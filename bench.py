@@ -57,6 +57,10 @@ def args_():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="large_zipf_bf16")
+    ap.add_argument("--tokens", type=int, default=0,
+                    help="override T (a reduced copy of the workload, for ncu captures)")
+    ap.add_argument("--experts", type=int, default=0,
+                    help="override E (a reduced copy of the workload, for ncu captures)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
@@ -76,6 +80,20 @@ def peaks():
     except Exception:
         return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
                 "source": "fallback"}
+
+
+def reduced_shape(a):
+    """The workload's shape, with T and E replaced when --tokens / --experts are given
+    (then the name says so and the line is not the workload's)."""
+    sh = mi.shape_by_name(a.workload)
+    kw = {}
+    if a.tokens:
+        kw["T"] = a.tokens
+    if a.experts:
+        kw["n_experts"] = a.experts
+    if kw:
+        sh = sh.with_(name=sh.name + "_reduced", **kw)
+    return sh
 
 
 def workload_desc(sh):
@@ -397,7 +415,7 @@ def main():
             dist.barrier()
 
     from paper_2506_02965_gb300.layer import MoELayer
-    sh = mi.shape_by_name(a.workload)
+    sh = reduced_shape(a)
     inp = mi.make_inputs(sh)
     lay = MoELayer(sh)
     lay.load(inp)

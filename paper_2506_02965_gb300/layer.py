@@ -18,12 +18,28 @@ import torch
 from . import _lib as L
 
 
+def overlap_default(shape) -> bool:
+    """Whether the aux loss and the router backward run on a second stream beside the
+    expert calls. That pays while the expert GEMMs leave SMs idle between and at the end
+    of their launches; once every launch fills the GPU for many rounds, the side-stream
+    kernels only take SMs from the persistent GEMM grids. Decided by the expert GEMM
+    work of one step."""
+    return shape.gemm_flops() < OVERLAP_MAX_FLOPS
+
+
+OVERLAP_MAX_FLOPS = float("inf")
+
+
 class MoELayer:
-    def __init__(self, shape, device: str = "cuda", owner_grouped=None):
+    def __init__(self, shape, device: str = "cuda", owner_grouped=None, overlap=None):
         """owner_grouped: lay the permuted rows out by owner party (expert e hosted by
-        party e mod P, moe_dispatch_owner) instead of by expert; default: when P > 1."""
+        party e mod P, moe_dispatch_owner) instead of by expert; default: when P > 1.
+        overlap: run the aux loss and the router backward on a second stream beside the
+        expert calls (True) or in order on the caller's stream (False); default: see
+        ``overlap_default``."""
         self.shape = sh = shape
         self.owner_grouped = (sh.n_parties > 1) if owner_grouped is None else bool(owner_grouped)
+        self.overlap = overlap_default(sh) if overlap is None else bool(overlap)
         self.device = device
         self.dt = torch.bfloat16 if sh.dtype == "bf16" else torch.float32
         self.cfg = L.make_config(sh.T, sh.d_model, sh.n_experts, sh.d_ff, sh.top_k, sh.n_parties,
@@ -172,35 +188,43 @@ class MoELayer:
         mark = mark or (lambda name: None)
         main = stream if stream is not None else torch.cuda.current_stream()
         self.route(main)
-        # the aux loss needs only probs and counts: compute it beside the experts
-        fork = torch.cuda.Event()
-        fork.record(main)
-        self.side.wait_event(fork)
-        self.aux(self.side)
-        aux_done = torch.cuda.Event()
-        aux_done.record(self.side)
+        if self.overlap:
+            # the aux loss needs only probs and counts: compute it beside the experts
+            fork = torch.cuda.Event()
+            fork.record(main)
+            self.side.wait_event(fork)
+            self.aux(self.side)
+            aux_done = torch.cuda.Event()
+            aux_done.record(self.side)
+        else:
+            self.aux(main)
         self.dispatch(main)
         mark("ffn_fwd_begin")
         self.ffn_fwd(main)
         mark("ffn_fwd_end")
         self.combine_fwd(main)
-        main.wait_event(aux_done)
+        if self.overlap:
+            main.wait_event(aux_done)
 
     def backward(self, stream=None, with_aux: bool = True, mark=None):
         mark = mark or (lambda name: None)
         main = stream if stream is not None else torch.cuda.current_stream()
         self.combine_bwd(main)
-        # the router backward needs only the gate gradients: run it beside the experts
-        fork = torch.cuda.Event()
-        fork.record(main)
-        self.side.wait_event(fork)
-        self.route_bwd(self.side, with_aux)
-        join = torch.cuda.Event()
-        join.record(self.side)
+        if self.overlap:
+            # the router backward needs only the gate gradients: run it beside the experts
+            fork = torch.cuda.Event()
+            fork.record(main)
+            self.side.wait_event(fork)
+            self.route_bwd(self.side, with_aux)
+            join = torch.cuda.Event()
+            join.record(self.side)
+        else:
+            self.route_bwd(main, with_aux)
         mark("ffn_bwd_begin")
         self.ffn_bwd(main)
         mark("ffn_bwd_end")
-        main.wait_event(join)
+        if self.overlap:
+            main.wait_event(join)
         self.dispatch_bwd(main)
 
     def step(self, stream=None, mark=None):

@@ -3,14 +3,25 @@
 Every floating-point comparison applies two bounds with the same rtol (the stated
 tolerance of the storage dtype):
   norm-wise:    max|gpu - ref| / max|ref| <= rtol
-  elementwise:  |gpu - ref| <= atol + rtol |ref| for every element, atol = rtol RMS(ref)
+  elementwise:  |gpu - ref| <= B (atol + rtol |ref|) for every element, atol = rtol RMS(ref)
 The norm-wise bound reads "max relative error" per tensor; the elementwise one also
-catches an error confined to the small-magnitude rows or columns of a tensor, which
-the norm-wise bound would let through. A stack of independent tensors (one weight
-gradient per expert, one router gradient per party) is compared slice by slice
-(assert_close_slices): each slice's own scale sets its bounds, so neither a small
-expert's error hides under a large expert's max nor a large expert's rounding is
-held to a small expert's RMS.
+catches an error confined to small-magnitude rows or elements, which the norm-wise
+bound would let through. A stack of independent tensors (one weight gradient per
+expert, one router gradient per party) is compared slice by slice
+(assert_close_slices): each slice's own maximum and RMS set its bounds, so a small
+expert's error cannot hide under a large expert's maximum, and a large expert's
+rounding is not held to the RMS of the small ones.
+
+B = 1, except for the end-to-end comparison of a bf16 run with the fp64 oracle, where
+B = 4. The bf16 path stores its saved activations and gradients (G, U, A, Y, dY, dH,
+dXp) in bf16 while the oracle keeps them exact, and the rows of one tensor differ in
+scale by the gate weights (more than 10x at k = 6). An element of a large-scale row
+whose sum cancels to near zero (dA = dY W2 for one feature, then dG, dU) inherits an
+absolute error of a few 2^-9 of its row's terms, which the tensor-wide RMS does not
+reflect: the worst such element measured 2.7 x the B = 1 bound (dh, k = 6), and a CPU
+emulation of the bf16 storage rounding (no GPU involved) reproduces the mechanism.
+Every GEMM and epilogue is also compared stage by stage, with the oracle given the
+GPU's own bf16 inputs of the stage, where B = 1.
 """
 import numpy as np
 
@@ -38,7 +49,7 @@ def rel_err(gpu, ref) -> float:
 
 def elem_ratio(gpu, ref, rtol) -> float:
     """max over elements of |g - r| / (atol + rtol |r|) with atol = rtol RMS(r); the
-    elementwise bound holds when this is <= 1 (0 for identical tensors)."""
+    elementwise bound holds when this is <= B (0 for identical tensors)."""
     g, r = np64(gpu), np.asarray(ref, np.float64)
     assert g.shape == r.shape, (g.shape, r.shape)
     if not r.size:
@@ -62,23 +73,30 @@ class Err(float):
         return f"{float(self):{spec}}/{self.elem:.2f}" if spec else f"{float(self)}/{self.elem:.2f}"
 
 
-def assert_close(name, gpu, ref, tol):
+# B of the elementwise bound for end-to-end comparisons against the fp64 oracle
+ELEM_B = {TOL["f32"]: 1.0, TOL["bf16"]: 4.0}
+
+
+def assert_close(name, gpu, ref, tol, stage=False):
+    """Both bounds (module doc). stage=True: the oracle was given the GPU's own inputs
+    of this stage, so B = 1 for every dtype."""
     e = rel_err(gpu, ref)
     assert e <= tol, f"{name}: max rel err {e:.3e} > {tol:.1e}"
     q = elem_ratio(gpu, ref, tol)
-    assert q <= 1.0, (f"{name}: elementwise |gpu-ref| exceeds {tol:.1e} (RMS(ref) + |ref|) "
-                      f"by a factor {q:.2f}")
+    b = 1.0 if stage else ELEM_B.get(tol, 1.0)
+    assert q <= b, (f"{name}: elementwise |gpu-ref| reaches {q:.2f} x {tol:.1e} (RMS(ref) + |ref|), "
+                    f"bound {b:.1f}")
     return Err(e, q)
 
 
-def assert_close_slices(name, gpu, ref, tol):
+def assert_close_slices(name, gpu, ref, tol, stage=False):
     """assert_close on every slice along the first axis; returns the worst slice's Err.
     A slice whose reference is all zero (an expert no token picked) must be exactly
     zero."""
     ref = np.asarray(ref, np.float64)
     worst = Err(0.0, 0.0)
     for i in range(ref.shape[0]):
-        e = assert_close(f"{name}[{i}]", gpu[i], ref[i], tol)
+        e = assert_close(f"{name}[{i}]", gpu[i], ref[i], tol, stage)
         worst = Err(max(float(e), float(worst)), max(e.elem, worst.elem))
     return worst
 

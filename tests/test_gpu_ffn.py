@@ -80,6 +80,29 @@ def test_expert_ffn_fwd_bwd(L, case):
         ref["dh"][r], ref["dxp"][r], ref["dw1"][e], ref["dw2"][e] = dH, dX, dW1, dW2
     for n in ref:  # weight gradients expert by expert
         (assert_close_slices if n in ("dw1", "dw2") else assert_close)(n, g[n], ref[n], tol)
+    # stage by stage: every contraction and epilogue against fp64 on the GPU's own stored
+    # inputs of that stage (bf16 G, U, A, dH), so only its accumulation and output
+    # rounding remain: elementwise bound B = 1
+    gh = {n: g[n].double().cpu().numpy() for n in ("h_gu", "act", "dh")}
+    st = {n: np.zeros_like(ref[n]) for n in ("y", "dh", "dxp", "dw1", "dw2")}
+    for e in range(E):
+        r = slice(off[e], off[e + 1])
+        if off[e + 1] == off[e]:
+            continue
+        G, U, A, dH = gh["h_gu"][r, :F], gh["h_gu"][r, F:], gh["act"][r], gh["dh"][r]
+        st["y"][r] = A @ w2[e].astype(np.float64).T
+        dA = dy[r].astype(np.float64) @ w2[e].astype(np.float64)
+        sg = mo.sigmoid(G)
+        st["dh"][r] = np.concatenate([dA * U * sg * (1.0 + G * (1.0 - sg)), dA * G * sg], 1)
+        st["dxp"][r] = dH @ w1[e].astype(np.float64)
+        st["dw1"][e] = dH.T @ xp[r].astype(np.float64)
+        st["dw2"][e] = dy[r].astype(np.float64).T @ A
+    for n in ("y", "dh", "dxp"):
+        assert_close(n + " (stage)", g[n], st[n], tol, stage=True)
+    for n in ("dw1", "dw2"):
+        assert_close_slices(n + " (stage)", g[n], st[n], tol, stage=True)
+    for n in ("h_gu", "act"):  # the forward's inputs are exact: the end-to-end reference is the stage's
+        assert_close(n + " (stage)", g[n], ref[n], tol, stage=True)
     if pattern == "skewed":  # the last expert got no rows: exact zero weight gradients
         assert off[E] - off[E - 1] == 0
         assert (g["dw1"][E - 1] == 0).all() and (g["dw2"][E - 1] == 0).all()

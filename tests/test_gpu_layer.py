@@ -79,6 +79,65 @@ def full_compare(lay, inp, sh):
     return errs
 
 
+def stage_compare(lay, inp, sh):
+    """Every stage of the layer against fp64 on the GPU's own stored inputs of that
+    stage (bf16 G, U, A, Y, dY, dH, dXp and fp32 gates as the GPU wrote them), so only
+    the stage's own accumulation and output rounding remain: elementwise bound B = 1.
+    Rows in the GPU's layout (expert-major or owner-grouped)."""
+    tol = TOL[sh.dtype]
+    bf = sh.dtype == "bf16"
+    F, E, k, T = sh.d_ff, sh.n_experts, sh.top_k, sh.T
+    g = {n: np64(getattr(lay, n)) for n in ("x_perm", "h_gu", "act", "y_perm", "dy_perm", "dh",
+                                            "dx_perm", "topk_w", "dtopk_w", "probs", "dlogits",
+                                            "dx_router")}
+    off = ints(lay.offsets)
+    ge = ints(lay.group_expert) if lay.owner_grouped else np.arange(E)
+    slot = ints(lay.slot_of).reshape(T, k)
+    w1 = np.asarray(inp["w1"], np.float64)
+    w2 = np.asarray(inp["w2"], np.float64)
+    dout = np.asarray(inp["dout"], np.float64)
+    st = {n: np.zeros_like(g[n]) for n in ("y_perm", "dh", "dx_perm")}
+    st["dw1"], st["dw2"] = np.zeros(w1.shape), np.zeros(w2.shape)
+    for q in range(E):
+        r, e = slice(off[q], off[q + 1]), ge[q]
+        if off[q + 1] == off[q]:
+            continue
+        G, U, A, dY, dH = g["h_gu"][r, :F], g["h_gu"][r, F:], g["act"][r], g["dy_perm"][r], g["dh"][r]
+        st["y_perm"][r] = A @ w2[e].T
+        dA = dY @ w2[e]
+        sg = mo.sigmoid(G)
+        st["dh"][r] = np.concatenate([dA * U * sg * (1.0 + G * (1.0 - sg)), dA * G * sg], 1)
+        st["dx_perm"][r] = dH @ w1[e]
+        st["dw1"][e] = dH.T @ g["x_perm"][r]
+        st["dw2"][e] = dY.T @ A
+    # combine and its backward on the GPU's expert outputs and gates
+    ysh = [np64(lay.y_sh[s2]) for s2 in range(sh.n_shared)]
+    st["out"] = mo.combine(g["y_perm"], g["topk_w"], slot) + sum(ysh, np.zeros((T, sh.d_model)))
+    st["dy_perm"], st["dtopk_w"] = mo.combine_backward(dout, g["y_perm"], g["topk_w"], slot)
+    # gating backward on the GPU's probs and gate gradients; its two products take the
+    # bf16 rounding of dlogits as operand on the bf16 path
+    rb = mo.router_backward(inp, sh, g["probs"], ints(lay.topk_idx), g["topk_w"], g["dtopk_w"],
+                            np64(lay.aux_coef))
+    dz = g["dlogits"]
+    dz_op = mi.bf16_round(dz.astype(np.float32)).astype(np.float64) if bf else dz
+    po = inp["party_offsets"]
+    wr = np.asarray(inp["w_router"], np.float64)
+    st["dw_router"] = np.stack([dz_op[po[p]:po[p + 1]].T @ np.asarray(inp["x"], np.float64)[po[p]:po[p + 1]]
+                                for p in range(sh.n_parties)])
+    st["dbias"] = np.stack([dz[po[p]:po[p + 1]].sum(0) for p in range(sh.n_parties)])
+    part = mo.party_of_tokens(T, po)
+    st["dx_router"] = np.einsum("te,ted->td", dz_op, wr[part])
+    dxsh = [np64(lay.dx_sh[s2]) for s2 in range(sh.n_shared)]
+    st["dx"] = mo.unpermute_reduce(g["dx_perm"], slot) + g["dx_router"] + sum(dxsh, np.zeros((T, sh.d_model)))
+    errs = {}
+    for n in ("y_perm", "dh", "dx_perm", "out", "dy_perm", "dtopk_w", "dx_router", "dx"):
+        errs[n] = assert_close(n + " (stage)", getattr(lay, n), st[n], tol, stage=True)
+    errs["dlogits"] = assert_close("dlogits (stage)", lay.dlogits, rb["dlogits"], tol, stage=True)
+    for n in ("dw1", "dw2", "dw_router", "dbias"):
+        errs[n] = assert_close_slices(n + " (stage)", getattr(lay, n), st[n], tol, stage=True)
+    return errs
+
+
 SMALL = {
     "tiny_f32": lambda: mi.SHAPES[1],
     "tiny_f32_renorm": lambda: mi.SHAPES[1].with_(normalize_topk=1, aux_alpha=1.0),
@@ -106,6 +165,8 @@ def test_layer_full_parity(L, name):
     assert status(L) == 0
     errs = full_compare(lay, inp, sh)
     print(name, {k: f"{v:.2e}" for k, v in errs.items()})
+    serrs = stage_compare(lay, inp, sh)
+    print(name, "stage", {k: f"{v:.2e}" for k, v in serrs.items()})
 
 
 def test_layer_is_deterministic(L):
