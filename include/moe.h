@@ -61,7 +61,7 @@ typedef enum { MOE_F32 = 0, MOE_BF16 = 1 } moe_dtype;
 typedef struct {
     int64_t T;              /* tokens in the batch (all parties) */
     int32_t d_model;        /* hidden size d */
-    int32_t n_experts;      /* E, global expert pool, 1..64 */
+    int32_t n_experts;      /* E, global expert pool, 1..256 (MOE_ERR_UNSUPPORTED above) */
     int32_t d_ff;           /* F, SwiGLU inner size of each routed expert */
     int32_t top_k;          /* k, 1..8, k <= E */
     int32_t n_parties;      /* P >= 1 */
@@ -323,8 +323,8 @@ moe_status moe_set_wait_limit_ns(uint64_t ns);
  *   MOE_PAIRS_ALL  (1): pair tiles for every such GEMM;
  *   MOE_PAIRS_AUTO (2, default): pair tiles for the input-gradient GEMM dX = dH W1
  *                   (contraction 2F) and wherever a launch has at least four rounds
- *                   of them, except under the SwiGLU backward epilogue (which, not the
- *                   operand feed, bounds the dA GEMM).
+ *                   of them, except under the SwiGLU backward epilogue when d < 2048
+ *                   (there the epilogue, not the operand feed, bounds the dA GEMM).
  * The weight-gradient GEMMs launched on their own (dW1; dW2 when dA runs as pairs; the
  * shared experts') follow the same mode with 256 x 256 output tiles where both output
  * dimensions are multiples of 256.

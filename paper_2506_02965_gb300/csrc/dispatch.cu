@@ -11,6 +11,7 @@
 namespace moe {
 
 constexpr int DCH = kDispatchChunkTokens;  // tokens per dispatch chunk (one thread each)
+constexpr int EMAX = 256;                  // experts (shared-memory tables below)
 
 // Per chunk: how many of its (token, pick) pairs went to each expert. Also checks
 // that every index lies in [0, E) and that no token picks an expert twice. With `send`
@@ -23,7 +24,7 @@ __global__ void __launch_bounds__(DCH) chunk_count_kernel(const int32_t* __restr
                                                           const int32_t* __restrict__ po, int P,
                                                           int32_t* send) {
     pdl_begin();
-    __shared__ int s_cnt[64];
+    __shared__ int s_cnt[EMAX];
     __shared__ int s_send[SEND_SMEM];
     const bool send_smem = send && P * P <= SEND_SMEM;
     for (int i = threadIdx.x; i < E; i += blockDim.x) s_cnt[i] = 0;
@@ -66,11 +67,12 @@ __global__ void __launch_bounds__(DCH) slot_kernel(const int32_t* __restrict__ i
                                                    int32_t* token_of, int Pown,
                                                    int32_t* group_expert) {
     pdl_begin();
-    __shared__ int s_pre[64];
-    __shared__ int s_tot[64];
-    __shared__ int s_base[64];
-    __shared__ unsigned s_bits[64][DCH / 32];
-    constexpr int TAB = 8192;  // chunk-count table staged in shared memory when it fits
+    __shared__ int s_pre[EMAX];
+    __shared__ int s_tot[EMAX];
+    __shared__ int s_base[EMAX];
+    __shared__ unsigned s_bits[EMAX][DCH / 32];
+    __shared__ int s_ppre[DCH], s_ptot[DCH];  // per (group, expert) partial sums
+    constexpr int TAB = 6144;  // chunk-count table staged in shared memory when it fits
     __shared__ int s_tab[TAB];
     const int c = blockIdx.x;
     const int64_t ntab = (int64_t)nchunks * E;
@@ -78,17 +80,47 @@ __global__ void __launch_bounds__(DCH) slot_kernel(const int32_t* __restrict__ i
         for (int i = threadIdx.x; i < ntab; i += blockDim.x) s_tab[i] = chunk_counts[i];
         __syncthreads();
     }
-    for (int e = threadIdx.x; e < E; e += blockDim.x) {
+    // per expert: the picks of the chunks before this one (pre) and of all chunks (tot).
+    // With E <= DCH the block's threads form G = DCH / E groups per expert, group g adding
+    // the chunks g, g + G, ...; the groups are then summed (integers: exact in any order).
+    auto cnt = [&](int cc, int e) {
+        return ntab <= TAB ? s_tab[cc * E + e] : chunk_counts[(int64_t)cc * E + e];
+    };
+    if (E <= DCH) {
+        const int G = DCH / E, e = threadIdx.x % E, g = threadIdx.x / E;
         int pre = 0, tot = 0;
-        for (int cc = 0; cc < nchunks; ++cc) {
-            const int v = ntab <= TAB ? s_tab[cc * E + e] : chunk_counts[(int64_t)cc * E + e];
-            if (cc < c) pre += v;
-            tot += v;
+        if (g < G) {
+            for (int cc = g; cc < nchunks; cc += G) {
+                const int v = cnt(cc, e);
+                if (cc < c) pre += v;
+                tot += v;
+            }
         }
-        s_pre[e] = pre;
-        s_tot[e] = tot;
+        s_ppre[threadIdx.x] = pre;
+        s_ptot[threadIdx.x] = tot;
+        __syncthreads();
+        if (threadIdx.x < E) {
+            int p2 = 0, t2 = 0;
+            for (int q = 0; q < G; ++q) {
+                p2 += s_ppre[q * E + threadIdx.x];
+                t2 += s_ptot[q * E + threadIdx.x];
+            }
+            s_pre[threadIdx.x] = p2;
+            s_tot[threadIdx.x] = t2;
+        }
+    } else {
+        for (int e = threadIdx.x; e < E; e += blockDim.x) {
+            int pre = 0, tot = 0;
+            for (int cc = 0; cc < nchunks; ++cc) {
+                const int v = cnt(cc, e);
+                if (cc < c) pre += v;
+                tot += v;
+            }
+            s_pre[e] = pre;
+            s_tot[e] = tot;
+        }
     }
-    for (int i = threadIdx.x; i < 64 * (DCH / 32); i += blockDim.x) (&s_bits[0][0])[i] = 0u;
+    for (int i = threadIdx.x; i < EMAX * (DCH / 32); i += blockDim.x) (&s_bits[0][0])[i] = 0u;
     __syncthreads();
     if (threadIdx.x == 0) {
         int run = 0, g = 0;

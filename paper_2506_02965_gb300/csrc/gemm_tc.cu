@@ -34,7 +34,7 @@ constexpr int EPI_BUF_BYTES = EPI_BOX * EPI_BOX * 2;
 constexpr int EPI_NBUF = 4;
 constexpr int EPI_STAGE_BYTES = EPI_NBUF * EPI_BUF_BYTES;
 __host__ __device__ constexpr int epi_stage_bytes(int) { return EPI_STAGE_BYTES; }
-constexpr int MAX_GROUPS = 128;
+constexpr int MAX_GROUPS = 256;
 
 struct Params {
     const int32_t* offsets;  // OFFSETS mode when non-null
@@ -53,6 +53,7 @@ struct Params {
     uint64_t wait_ns;
     // EPI_ROUTE: out0 = logits, out1 = probs (fp32 [T,E]), aux = bias [P,E] or null
     int E, k, normalize, hist_n;
+    int band;  // tile order: bands of `band` M-tiles, each swept along N (set at launch)
     int32_t* topk_idx;
     float* topk_w;
     int32_t* counts;
@@ -403,6 +404,105 @@ __device__ __forceinline__ void route_epilogue(const Params& p, const Tile& ti, 
     }
 }
 
+// Gating of Alg. 7 for E > 64 (BN = 128 or 256 accumulator columns): the same results
+// as route_epilogue without holding all logits in registers. The accumulator stays in
+// TMEM, read 32 columns at a time in three passes: (1) bias, logits out, running max and
+// the k largest logits by insertion into a sorted list (ids arrive in ascending order
+// and only a strictly larger logit moves ahead, so equal logits keep the lower id
+// first); (2) the sum of exp(z - max); (3) the probabilities. Logits and probabilities
+// are written element by element (any E). Every lane runs the TMEM loads (they are
+// warp-collective); only valid rows use them.
+template <int BN>
+__device__ __forceinline__ void route_epilogue_wide(const Params& p, const Tile& ti, int m, bool valid,
+                                                    uint32_t tbase, int* hist) {
+    const int E = p.E, k = p.k;
+    const int64_t t = ti.out_row + m;
+    const float* bias = (const float*)p.aux;
+    float* lg = (float*)p.out0 + t * E;
+    float* pr = (float*)p.out1 + t * E;
+    float mx = -3.402823466e38f;
+    float tv[8];
+    int tid[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+        tv[j] = -3.402823466e38f;
+        tid[j] = -1;
+    }
+#pragma unroll 1
+    for (int c = 0; c < BN; c += 32) {
+        float z[32];
+        tmem_ld32(tbase + c, z);
+        if (valid) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+                const int e = c + i;
+                if (e < E) {
+                    float v = z[i] + (bias ? bias[ti.g * E + e] : 0.f);
+                    lg[e] = v;
+                    mx = fmaxf(mx, v);
+                    // insert at the first slot that is empty or holds a smaller logit,
+                    // then shift the rest down by one
+                    float cv = v;
+                    int ce = e;
+                    bool shifting = false;
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) {
+                        if (j < k && (shifting || tid[j] < 0 || cv > tv[j])) {
+                            const float tvj = tv[j];
+                            const int tij = tid[j];
+                            tv[j] = cv;
+                            tid[j] = ce;
+                            cv = tvj;
+                            ce = tij;
+                            shifting = true;
+                            if (ce < 0) break;
+                        }
+                    }
+                }
+            }
+        }
+    }
+    float sum = 0.f;
+#pragma unroll 1
+    for (int c = 0; c < BN; c += 32) {
+        float z[32];
+        tmem_ld32(tbase + c, z);
+        if (valid) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i)
+                if (c + i < E) sum += expf(z[i] + (bias ? bias[ti.g * E + c + i] : 0.f) - mx);
+        }
+    }
+#pragma unroll 1
+    for (int c = 0; c < BN; c += 32) {
+        float z[32];
+        tmem_ld32(tbase + c, z);
+        if (valid) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i)
+                if (c + i < E) pr[c + i] = expf(z[i] + (bias ? bias[ti.g * E + c + i] : 0.f) - mx) / sum;
+        }
+    }
+    if (!valid) return;
+    float wsel[8], wsum = 0.f;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+        wsel[j] = 0.f;
+        if (j < k) {
+            wsel[j] = expf(tv[j] - mx) / sum;
+            wsum += wsel[j];
+        }
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+        if (j < k) {
+            p.topk_idx[t * k + j] = tid[j];
+            p.topk_w[t * k + j] = p.normalize ? wsel[j] / wsum : wsel[j];
+            atomicAdd(&hist[ti.g * E + tid[j]], 1);
+        }
+    }
+}
+
 // ------------------------------------------------------------------------ the kernel
 // PAIR: the two CTAs of a cluster compute one 256 x BN tile with tcgen05 cta_group::2
 // MMAs issued by CTA 0: each CTA holds 128 rows of A and BN/2 rows of B in its own
@@ -445,7 +545,6 @@ __global__ void __launch_bounds__(THREADS, 1)
     __shared__ int s_tile_start[MAX_GROUPS + 1];
     __shared__ int s_total1;  // fused: tiles of the first problem
     __shared__ unsigned char s_order[DW2 ? MAX_GROUPS : 1];  // fused: second problem's group order
-    __shared__ int s_rows[DW2 ? MAX_GROUPS : 1];
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     volatile int* abort_flag = &s_abort;
@@ -472,18 +571,19 @@ __global__ void __launch_bounds__(THREADS, 1)
         if constexpr (DW2) s_tile_start[p.G] = acc + p.G * (p2.Mout / BM) * (p2.N / BN);
         s_abort = 0;
     }
-    if constexpr (DW2) {
-        for (int g = threadIdx.x; g < p2.G; g += blockDim.x) s_rows[g] = p2.offsets[g + 1] - p2.offsets[g];
-    }
     __syncthreads();
     if constexpr (DW2) {
         // weight-gradient groups longest first (each tile of a group runs over all its
         // rows): with skewed experts the long tiles then do not form the tail. Rank of g =
-        // groups with more rows, or as many and a lower index.
+        // groups with more rows, or as many and a lower index. (Row counts are read from
+        // the offsets in global memory: static shared memory is at its limit here.)
         for (int g = threadIdx.x; g < p2.G; g += blockDim.x) {
+            const int rg = p2.offsets[g + 1] - p2.offsets[g];
             int rank = 0;
-            for (int h = 0; h < p2.G; ++h)
-                rank += (s_rows[h] > s_rows[g]) || (s_rows[h] == s_rows[g] && h < g);
+            for (int h = 0; h < p2.G; ++h) {
+                const int rh = p2.offsets[h + 1] - p2.offsets[h];
+                rank += (rh > rg) || (rh == rg && h < g);
+            }
             s_order[rank] = (unsigned char)g;
         }
         __syncthreads();
@@ -491,6 +591,21 @@ __global__ void __launch_bounds__(THREADS, 1)
     const int total_tiles = s_tile_start[p.G];
     if (tile0 >= total_tiles) return;  // uniform across the pair
 
+    // Tile order inside a group: bands of `band` M-tiles, each band swept along N with
+    // the M-tiles of the band innermost. The tiles that run at the same time (one round
+    // of the persistent grid, C of them) then cover about band x C/band output tiles and
+    // read band A blocks and C/band B blocks, instead of one A block and C B blocks when
+    // whole rows of N-tiles come first (band ~ sqrt(C) minimises the blocks per round;
+    // the A blocks of a band also stay in L2 while it sweeps N).
+    auto band_split = [&](int local, int mt_g, int nt_g, int band, int* mt, int* nt) {
+        const int gmx = band > 0 ? band : 1;
+        const int b = local / (gmx * nt_g);
+        const int first = b * gmx;
+        const int gm = min(gmx, mt_g - first);
+        const int rem = local - b * gmx * nt_g;
+        *mt = first + rem % gm;
+        *nt = rem / gm;
+    };
     auto tile_at = [&](int t) -> Tile {
         Tile ti;
         ti.dw = false;
@@ -499,11 +614,13 @@ __global__ void __launch_bounds__(THREADS, 1)
                 const int per = (p2.Mout / BM) * (p2.N / BN);
                 const int g = s_order[(t - s_total1) / per], l2 = (t - s_total1) % per;
                 const int tn2 = p2.N / BN;
+                int mt2, nt2;
+                band_split(l2, p2.Mout / BM, tn2, p2.band, &mt2, &nt2);
                 ti.dw = true;
                 ti.g = g;
                 ti.we = p2.gexp ? p2.gexp[g] : g;
-                ti.m0 = (l2 / tn2) * BM;
-                ti.n0 = (l2 % tn2) * BN;
+                ti.m0 = mt2 * BM;
+                ti.n0 = nt2 * BN;
                 const int64_t r0 = p2.offsets[g], nrows = p2.offsets[g + 1] - r0;
                 ti.mvalid = p2.Mout;
                 ti.a_row = ti.b_row = r0;
@@ -513,10 +630,19 @@ __global__ void __launch_bounds__(THREADS, 1)
                 return ti;
             }
         }
-        int g = 0;
-        while (g + 1 < p.G && s_tile_start[g + 1] <= t) ++g;
+        // the group whose tile range holds t: last g with s_tile_start[g] <= t (binary
+        // search; empty groups share their start with the next one)
+        int lo = 0, hi = p.G - 1;
+        while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1;
+            if (s_tile_start[mid] <= t) lo = mid;
+            else hi = mid - 1;
+        }
+        const int g = lo;
         const int local = t - s_tile_start[g];
-        const int mt = local / tiles_n, nt = local % tiles_n;
+        const int g_end = (g + 1 < p.G) ? s_tile_start[g + 1] : s_total1;
+        int mt, nt;
+        band_split(local, (g_end - s_tile_start[g]) / tiles_n, tiles_n, p.band, &mt, &nt);
         ti.g = g;
         ti.we = p.gexp ? p.gexp[g] : g;
         ti.m0 = mt * BMP + (int)rank * BM;
@@ -1039,7 +1165,11 @@ __global__ void __launch_bounds__(THREADS, 1)
                         emit(3, vals, maps, cols, direct);
                     }
                 } else if constexpr (EPI == EPI_ROUTE) {
-                    route_epilogue<BN>(p, ti, m, valid, tbase, route_hist);
+                    // the per-(party, expert) counts: a shared-memory histogram when P E fits
+                    // (hist_n > 0), else straight to the global counts
+                    int* hist = p.hist_n ? route_hist : p.counts;
+                    if constexpr (BN <= 64) route_epilogue<BN>(p, ti, m, valid, tbase, hist);
+                    else route_epilogue_wide<BN>(p, ti, m, valid, tbase, hist);
                 } else if constexpr (EPI == EPI_DWR) {
                     // one token chunk's partial router gradient: accumulator row m is model
                     // column m, column e is expert e; stored transposed, fp32, part[g][e][m]
@@ -1175,6 +1305,14 @@ static int sm_count() {
     return n;
 }
 
+// M-tiles per band of the tile order for `c` tiles in flight at once (the persistent
+// CTAs, or CTA pairs): about sqrt(c).
+static int band_for(int c) {
+    int b = 1;
+    while ((b + 1) * (b + 1) <= c) ++b;
+    return b;
+}
+
 template <int BN, bool B_MN, bool VAR_K, int EPI, bool PAIR = false, bool DW2 = false>
 static cudaError_t launch(const CUtensorMap& ma, const CUtensorMap& mb, const CUtensorMap& mo0,
                           const CUtensorMap& mo1, const Params& p, int64_t tiles_ub,
@@ -1185,7 +1323,8 @@ static cudaError_t launch(const CUtensorMap& ma, const CUtensorMap& mb, const CU
     const CUtensorMap& A2 = ma2 ? *ma2 : ma;
     const CUtensorMap& B2 = mb2 ? *mb2 : mb;
     const CUtensorMap& O2 = mo2 ? *mo2 : mo0;
-    const Params& P2 = p2 ? *p2 : p;
+    Params P1 = p;
+    Params P2 = p2 ? *p2 : p;
     constexpr int NPAIR = PAIR ? 2 : 1;
     constexpr int NST = num_stages((uint32_t)(BM * BK * 2 + BN / NPAIR * BK * 2), EPI);
     const int extra_max = EPI == EPI_ROUTE ? 64 * 64 * 4 : EPI_WARPS * epi_stage_bytes(EPI);
@@ -1223,6 +1362,7 @@ static cudaError_t launch(const CUtensorMap& ma, const CUtensorMap& mb, const CU
             max_clusters = n;
         }
         const int clusters = (int)std::min<int64_t>(tiles_ub, max_clusters);
+        P1.band = P2.band = band_for(clusters);
         cudaLaunchConfig_t cfg = {};
         cfg.gridDim = dim3(2 * clusters);
         cfg.blockDim = dim3(THREADS);
@@ -1237,10 +1377,11 @@ static cudaError_t launch(const CUtensorMap& ma, const CUtensorMap& mb, const CU
         attr[1].val.programmaticStreamSerializationAllowed = 1;
         cfg.attrs = attr;
         cfg.numAttrs = 2;
-        return cudaLaunchKernelEx(&cfg, kern, ma, mb, mo0, mo1, p, A2, B2, O2, P2);
+        return cudaLaunchKernelEx(&cfg, kern, ma, mb, mo0, mo1, P1, A2, B2, O2, P2);
     } else {
         const int grid = (int)std::min<int64_t>(tiles_ub, sm_count());
-        (void)launch_pdl(kern, dim3(grid), dim3(THREADS), smem, s, ma, mb, mo0, mo1, p, A2, B2, O2, P2);
+        P1.band = P2.band = band_for(grid);
+        (void)launch_pdl(kern, dim3(grid), dim3(THREADS), smem, s, ma, mb, mo0, mo1, P1, A2, B2, O2, P2);
         return cudaGetLastError();
     }
 }
@@ -1256,12 +1397,16 @@ void set_gemm_pairs(int mode) { tc::g_pairs = mode; }
 // pairs with fewer tiles too: an SM ingests at most ~145 GB/s from L2 with TMA, which
 // caps a single-CTA 128 x 256 tile near 80% of the MMA rate and a pair's 256 x 256 tile
 // (half the B bytes per SM) does not, and its weight-gradient partner then runs beside
-// it on the second stream.
+// it on the second stream. The SwiGLU-backward GEMM (dA) moves G, U, dG and dU in its
+// epilogue: with a short contraction (d < 2048) the epilogue bounds it and single-CTA
+// tiles fused with dW2 in one launch are faster; from d = 2048 the mainloop dominates
+// and pairs win (d = 4096: the expert backward 17.8 -> 17.2 ms; d = 1024: +4%).
 bool gemm_m_uses_pairs(const GemmMArgs& g) {
     using namespace tc;
     if (g.N % 256 != 0) return false;
     if (g_pairs == MOE_PAIRS_ALL) return true;
-    if (g_pairs != MOE_PAIRS_AUTO || g.epi == EPI_SWIGLU_BWD) return false;
+    if (g_pairs != MOE_PAIRS_AUTO) return false;
+    if (g.epi == EPI_SWIGLU_BWD && g.K < 2048) return false;
     if (g.epi == EPI_STORE && !g.b_kmajor && g.K >= 512) return true;
     const int64_t pt_ub = g.rows.offsets ? ((int64_t)g.rows.rows + 2 * BM - 1) / (2 * BM) + g.G
                                          : (int64_t)g.G * ((g.rows.rows + 2 * BM - 1) / (2 * BM));
@@ -1381,10 +1526,12 @@ cudaError_t launch_gemm_k(const GemmKArgs& g, bool bf16, cudaStream_t s) {
     if (!make_map(&ma, g.a, g.M, rows_a, 64)) return cudaErrorInvalidValue;
     if (!make_map(&mb, g.b, g.N, rows_b, 64)) return cudaErrorInvalidValue;
     const int64_t tiles = (int64_t)g.G * (g.M / BM);
-    if (g.epi == EPI_DWR) {  // fp32 partials, N = 64 (experts, zero-padded)
-        if (g.N != 64 || g.M % BM) return cudaErrorInvalidValue;
+    if (g.epi == EPI_DWR) {  // fp32 partials, N = 64, 128 or 256 (experts, zero-padded)
+        if ((g.N != 64 && g.N != 128 && g.N != 256) || g.M % BM) return cudaErrorInvalidValue;
         p.E = g.E;
-        return launch<64, true, true, EPI_DWR>(ma, mb, ma, ma, p, tiles, s);
+        if (g.N == 64) return launch<64, true, true, EPI_DWR>(ma, mb, ma, ma, p, tiles, s);
+        if (g.N == 128) return launch<128, true, true, EPI_DWR>(ma, mb, ma, ma, p, tiles, s);
+        return launch<256, true, true, EPI_DWR>(ma, mb, ma, ma, p, tiles, s);
     }
     if (!make_map(&mo, g.out, g.N, (int64_t)g.G * g.M, 0, true)) return cudaErrorInvalidValue;
     if (gemm_k_uses_pairs(g))
@@ -1469,7 +1616,7 @@ cudaError_t launch_route_tc(const RouteArgs& a, cudaStream_t s) {
     p.E = a.E;
     p.k = a.k;
     p.normalize = a.normalize;
-    p.hist_n = a.P * a.E;
+    p.hist_n = a.P * a.E <= 64 * 64 ? a.P * a.E : 0;  // else counted in global memory
     p.out0 = a.logits;
     p.out1 = a.probs;
     p.aux = a.bias;
@@ -1478,7 +1625,8 @@ cudaError_t launch_route_tc(const RouteArgs& a, cudaStream_t s) {
     p.counts = a.counts;
     p.b_group_rows = a.E;
     p.wait_ns = g_wait_ns;
-    const int BNr = a.E <= 16 ? 16 : a.E <= 32 ? 32 : 64;
+    const int BNr = a.E <= 16 ? 16 : a.E <= 32 ? 32 : a.E <= 64 ? 64 : a.E <= 128 ? 128 : 256;
+    if (a.E > 256) return cudaErrorInvalidValue;
     p.N = BNr;
     CUtensorMap ma, mb;
     if (!make_map(&ma, a.x, a.d, a.T, BM)) return cudaErrorInvalidValue;
@@ -1486,7 +1634,9 @@ cudaError_t launch_route_tc(const RouteArgs& a, cudaStream_t s) {
     const int64_t tiles = (a.T + BM - 1) / BM + a.P;
     if (BNr == 16) return launch<16, false, false, EPI_ROUTE>(ma, mb, ma, ma, p, tiles, s);
     if (BNr == 32) return launch<32, false, false, EPI_ROUTE>(ma, mb, ma, ma, p, tiles, s);
-    return launch<64, false, false, EPI_ROUTE>(ma, mb, ma, ma, p, tiles, s);
+    if (BNr == 64) return launch<64, false, false, EPI_ROUTE>(ma, mb, ma, ma, p, tiles, s);
+    if (BNr == 128) return launch<128, false, false, EPI_ROUTE>(ma, mb, ma, ma, p, tiles, s);
+    return launch<256, false, false, EPI_ROUTE>(ma, mb, ma, ma, p, tiles, s);
 }
 
 cudaError_t gemm_status(cudaStream_t s, int* code) { return tu_status_read_clear(s, code); }

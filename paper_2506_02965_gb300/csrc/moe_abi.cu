@@ -42,8 +42,11 @@ moe_status check_cfg(const moe_config* c) {
     if (c->T < 0) return fail(MOE_ERR_INVALID_ARG, "T=%lld < 0", (long long)c->T);
     if (c->d_model <= 0 || c->d_ff <= 0)
         return fail(MOE_ERR_INVALID_ARG, "d_model=%d and d_ff=%d must be > 0", c->d_model, c->d_ff);
-    if (c->n_experts < 1 || c->n_experts > 64)
-        return fail(MOE_ERR_INVALID_ARG, "n_experts=%d outside [1,64]", c->n_experts);
+    if (c->n_experts < 1)
+        return fail(MOE_ERR_INVALID_ARG, "n_experts=%d < 1", c->n_experts);
+    if (c->n_experts > 256)
+        return fail(MOE_ERR_UNSUPPORTED, "n_experts=%d > 256, the largest expert pool this build handles",
+                    c->n_experts);
     if (c->top_k < 1 || c->top_k > 8 || c->top_k > c->n_experts)
         return fail(MOE_ERR_INVALID_ARG, "top_k=%d outside [1, min(8, E)]", c->top_k);
     if (c->n_parties < 1 || c->n_parties > 64)

@@ -15,31 +15,46 @@ namespace moe {
 namespace cg = cooperative_groups;
 
 // ----------------------------------------------------------------------------- top-k
-// Per token, lane l owns experts l and l + 32 (E <= 64). Picks the k largest logits,
-// descending, equal logits by ascending expert id; writes logits (optional), probs,
-// topk idx / w and bumps the block histogram.
+// Per token, lane l owns experts l + 32 i, i < NV (E <= 32 NV). Picks the k largest
+// logits, descending, equal logits by ascending expert id; writes logits (optional),
+// probs, topk idx / w and bumps the block histogram (or the global counts when the
+// histogram does not fit in shared memory).
 __device__ __forceinline__ bool better(float va, int ia, float vb, int ib) {
     return va > vb || (va == vb && ia < ib);
 }
 
-__device__ void softmax_topk_token(float z0, float z1, int lane, int E, int k, int normalize,
+template <int NV>
+__device__ void softmax_topk_token(const float (&z)[NV], int lane, int E, int k, int normalize,
                                    int64_t t, int party, float* logits, float* probs,
                                    int32_t* topk_idx, float* topk_w, int* s_hist) {
-    const int e0 = lane, e1 = lane + 32;
-    const bool v0 = e0 < E, v1 = e1 < E;
-    if (logits) {
-        if (v0) logits[t * E + e0] = z0;
-        if (v1) logits[t * E + e1] = z1;
+    bool val[NV], taken[NV];
+#pragma unroll
+    for (int i = 0; i < NV; ++i) {
+        val[i] = lane + 32 * i < E;
+        taken[i] = !val[i];
     }
-    float m = fmaxf(v0 ? z0 : -FLT_MAX, v1 ? z1 : -FLT_MAX);
+    if (logits) {
+#pragma unroll
+        for (int i = 0; i < NV; ++i)
+            if (val[i]) logits[t * E + lane + 32 * i] = z[i];
+    }
+    float m = -FLT_MAX;
+#pragma unroll
+    for (int i = 0; i < NV; ++i) m = fmaxf(m, val[i] ? z[i] : -FLT_MAX);
     m = warp_max(m);
-    float x0 = v0 ? expf(z0 - m) : 0.f;
-    float x1 = v1 ? expf(z1 - m) : 0.f;
-    float s = warp_sum(x0 + x1);
-    float p0 = x0 / s, p1 = x1 / s;
-    if (v0) probs[t * E + e0] = p0;
-    if (v1) probs[t * E + e1] = p1;
-    bool taken0 = !v0, taken1 = !v1;
+    float x[NV], loc = 0.f;
+#pragma unroll
+    for (int i = 0; i < NV; ++i) {
+        x[i] = val[i] ? expf(z[i] - m) : 0.f;
+        loc += x[i];
+    }
+    const float s = warp_sum(loc);
+    float p[NV];
+#pragma unroll
+    for (int i = 0; i < NV; ++i) {
+        p[i] = x[i] / s;
+        if (val[i]) probs[t * E + lane + 32 * i] = p[i];
+    }
     float wsel = 0.f, wsum = 0.f;
     int isel = 0;
     for (int j = 0; j < k; ++j) {
@@ -47,8 +62,14 @@ __device__ void softmax_topk_token(float z0, float z1, int lane, int E, int k, i
         float cv = -FLT_MAX;
         int ci = 0x7fffffff;
         bool have = false;
-        if (!taken0) { cv = z0; ci = e0; have = true; }
-        if (!taken1 && (!have || better(z1, e1, cv, ci))) { cv = z1; ci = e1; have = true; }
+#pragma unroll
+        for (int i = 0; i < NV; ++i) {
+            if (!taken[i] && (!have || better(z[i], lane + 32 * i, cv, ci))) {
+                cv = z[i];
+                ci = lane + 32 * i;
+                have = true;
+            }
+        }
         int hv = have ? 1 : 0;
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) {
@@ -57,11 +78,16 @@ __device__ void softmax_topk_token(float z0, float z1, int lane, int E, int k, i
             int oh = __shfl_xor_sync(0xffffffffu, hv, o);
             if (oh && (!hv || better(ov, oi, cv, ci))) { cv = ov; ci = oi; hv = 1; }
         }
-        // ci is the winner on every lane
-        const int owner = ci & 31;
-        float pw = __shfl_sync(0xffffffffu, (ci < 32) ? p0 : p1, owner);
-        if (ci == e0) taken0 = true;
-        if (ci == e1) taken1 = true;
+        // ci is the winner on every lane; its owner lane holds its probability
+        const int owner = ci & 31, slot = ci >> 5;
+        float mine = 0.f;
+#pragma unroll
+        for (int i = 0; i < NV; ++i)
+            if (i == slot) mine = p[i];
+        const float pw = __shfl_sync(0xffffffffu, mine, owner);
+#pragma unroll
+        for (int i = 0; i < NV; ++i)
+            if (ci == lane + 32 * i) taken[i] = true;
         if (lane == j) { isel = ci; wsel = pw; }
         wsum += pw;
         if (lane == 0) atomicAdd(&s_hist[party * E + ci], 1);
@@ -76,15 +102,26 @@ __device__ void softmax_topk_token(float z0, float z1, int lane, int E, int k, i
 // One warp handles a group of up to TPW consecutive tokens of one party. Lane l
 // accumulates the dot products of its 16-byte column chunks for every expert, then
 // the partial sums are combined with a butterfly (identical bits on every lane).
+// FROM_LOGITS: the logits come from logits_in instead ([T,E] fp32); with a bias they
+// are the router's raw products (E > 64, computed by a GEMM): the bias is added here
+// and the biased logits are written back to `logits` (which may be logits_in).
+// The per-(party, expert) counts go through a shared-memory histogram when P E fits
+// (HIST_SMEM), else straight to the global counts.
+constexpr int HIST_SMEM = 4096;
 template <typename T, int EMAX, int TPW, bool FROM_LOGITS>
 __global__ void __launch_bounds__(256) route_kernel(
     const T* __restrict__ x, const T* __restrict__ wr, const float* __restrict__ bias,
-    const float* __restrict__ logits_in, const int32_t* __restrict__ po, int P, int64_t Tn,
+    const float* logits_in, const int32_t* __restrict__ po, int P, int64_t Tn,
     int d, int E, int k, int normalize, float* logits, float* probs, int32_t* topk_idx,
     float* topk_w, int32_t* counts) {
     pdl_begin();
-    extern __shared__ int s_hist[];  // [P*E]
-    for (int i = threadIdx.x; i < P * E; i += blockDim.x) s_hist[i] = 0;
+    constexpr int NV = (EMAX + 31) / 32;
+    extern __shared__ int s_hist_dyn[];  // [P*E] when it fits
+    const bool hist_smem = P * E <= HIST_SMEM;
+    int* s_hist = hist_smem ? s_hist_dyn : counts;
+    if (hist_smem) {
+        for (int i = threadIdx.x; i < P * E; i += blockDim.x) s_hist[i] = 0;
+    }
     __syncthreads();
     using V = Vec<T>;
     constexpr int VN = V::N;
@@ -108,13 +145,16 @@ __global__ void __launch_bounds__(256) route_kernel(
             g -= ng;
         }
         const int n = (int)min64(TPW, tend - t0);
-        float z0[TPW], z1[TPW];
+        float z[TPW][NV];
         if constexpr (FROM_LOGITS) {
 #pragma unroll
-            for (int i = 0; i < TPW; ++i) {
-                z0[i] = (i < n && lane < E) ? logits_in[(t0 + i) * E + lane] : 0.f;
-                z1[i] = (i < n && lane + 32 < E) ? logits_in[(t0 + i) * E + lane + 32] : 0.f;
-            }
+            for (int i = 0; i < TPW; ++i)
+#pragma unroll
+                for (int v = 0; v < NV; ++v) {
+                    const int e = lane + 32 * v;
+                    z[i][v] = (i < n && e < E) ? logits_in[(t0 + i) * E + e] : 0.f;
+                    if (bias && e < E) z[i][v] += bias[party * E + e];
+                }
         } else {
             float acc[TPW][EMAX];
 #pragma unroll
@@ -146,30 +186,34 @@ __global__ void __launch_bounds__(256) route_kernel(
             }
 #pragma unroll
             for (int i = 0; i < TPW; ++i) {
-                z0[i] = 0.f;
-                z1[i] = 0.f;
+#pragma unroll
+                for (int v = 0; v < NV; ++v) z[i][v] = 0.f;
 #pragma unroll
                 for (int e = 0; e < EMAX; ++e) {
                     float s = warp_sum(acc[i][e]);
-                    if (e == lane) z0[i] = s;
-                    if (e == lane + 32) z1[i] = s;
+#pragma unroll
+                    for (int v = 0; v < NV; ++v)
+                        if (e == lane + 32 * v) z[i][v] = s;
                 }
                 if (bias) {
-                    if (lane < E) z0[i] += bias[party * E + lane];
-                    if (lane + 32 < E) z1[i] += bias[party * E + lane + 32];
+#pragma unroll
+                    for (int v = 0; v < NV; ++v)
+                        if (lane + 32 * v < E) z[i][v] += bias[party * E + lane + 32 * v];
                 }
             }
         }
 #pragma unroll
         for (int i = 0; i < TPW; ++i)
             if (i < n)
-                softmax_topk_token(z0[i], z1[i], lane, E, k, normalize, t0 + i, party,
-                                   FROM_LOGITS ? nullptr : logits, probs, topk_idx, topk_w,
-                                   s_hist);
+                softmax_topk_token<NV>(z[i], lane, E, k, normalize, t0 + i, party,
+                                       (FROM_LOGITS && !bias) ? nullptr : logits, probs, topk_idx,
+                                       topk_w, s_hist);
     }
     __syncthreads();
-    for (int i = threadIdx.x; i < P * E; i += blockDim.x)
-        if (s_hist[i]) atomicAdd(&counts[i], s_hist[i]);
+    if (hist_smem) {
+        for (int i = threadIdx.x; i < P * E; i += blockDim.x)
+            if (s_hist[i]) atomicAdd(&counts[i], s_hist[i]);
+    }
 }
 
 // ----------------------------------------------------------------------------- aux loss
@@ -186,7 +230,7 @@ __global__ void __cluster_dims__(AUX_CLUSTER, 1, 1) __launch_bounds__(AUX_THREAD
                     float* loss, float* coef) {
     pdl_begin();
     __shared__ float s_part[AUX_THREADS];
-    __shared__ float s_col[64];
+    __shared__ float s_col[256];
     cg::cluster_group cluster = cg::this_cluster();
     const int rank = (int)cluster.block_rank();
     const int p = blockIdx.x / AUX_CLUSTER;
@@ -252,15 +296,17 @@ __device__ __forceinline__ bool chunk_of(int64_t ci, const int32_t* po, int P, i
 }
 
 // dlogits, one warp per token (Alg. 7 backward with the picks held fixed); lane l
-// holds experts l and l + 32. For the tensor-core router gradients it also writes
-// dz16 [T, 64], dlogits rounded to bf16 with zero columns past E, and (block 0) the
-// token chunks of the chunked dW_r contraction: chunk_off[c] = first token of chunk c,
-// the chunks of CH tokens of each party in order, then empty chunks up to nchunk.
+// holds experts l + 32 i, i < NV. For the tensor-core router gradients it also writes
+// dz16 [T, EP], dlogits rounded to bf16 with zero columns past E (EP = E rounded up to
+// 64, 128 or 256), and (block 0) the token chunks of the chunked dW_r contraction:
+// chunk_off[c] = first token of chunk c, the chunks of CH tokens of each party in
+// order, then empty chunks up to nchunk.
+template <int NV>
 __global__ void __launch_bounds__(256) dlogits_kernel(
     const float* __restrict__ probs, const int32_t* __restrict__ topk_idx,
     const float* __restrict__ topk_w, const float* __restrict__ dtopk_w,
     const float* __restrict__ aux_coef, const int32_t* __restrict__ po, int P, int64_t Tn, int E,
-    int k, int normalize, float* dlogits, __nv_bfloat16* dz16, int32_t* chunk_off, int CH,
+    int k, int normalize, float* dlogits, __nv_bfloat16* dz16, int EP, int32_t* chunk_off, int CH,
     int nchunk) {
     pdl_begin();
     const int lane = threadIdx.x & 31;
@@ -275,9 +321,13 @@ __global__ void __launch_bounds__(256) dlogits_kernel(
     }
     if (t >= Tn) return;
     const int party = party_of(po, P, t);
-    const int e0 = lane, e1 = lane + 32;
-    const float p0 = e0 < E ? probs[t * E + e0] : 0.f;
-    const float p1 = e1 < E ? probs[t * E + e1] : 0.f;
+    float p[NV], dp[NV];
+#pragma unroll
+    for (int i = 0; i < NV; ++i) {
+        const int e = lane + 32 * i;
+        p[i] = e < E ? probs[t * E + e] : 0.f;
+        dp[i] = (aux_coef && e < E) ? aux_coef[party * E + e] : 0.f;
+    }
     // lane j < k holds pick j
     const int ej = lane < k ? topk_idx[t * k + lane] : -1;
     const float gj0 = lane < k ? dtopk_w[t * k + lane] : 0.f;
@@ -288,21 +338,23 @@ __global__ void __launch_bounds__(256) dlogits_kernel(
         const float S = warp_sum((ej >= 0 && ej < E) ? probs[t * E + ej] : 0.f);
         gj = (gj0 - inner) / S;
     }
-    float dp0 = (aux_coef && e0 < E) ? aux_coef[party * E + e0] : 0.f;
-    float dp1 = (aux_coef && e1 < E) ? aux_coef[party * E + e1] : 0.f;
     for (int j = 0; j < k; ++j) {
         const int e = __shfl_sync(0xffffffffu, ej, j);
         const float g = __shfl_sync(0xffffffffu, gj, j);
-        if (e == e0) dp0 += g;
-        if (e == e1) dp1 += g;
+#pragma unroll
+        for (int i = 0; i < NV; ++i)
+            if (e == lane + 32 * i) dp[i] += g;
     }
-    const float dot = warp_sum(dp0 * p0 + dp1 * p1);
-    const float z0 = p0 * (dp0 - dot), z1 = p1 * (dp1 - dot);
-    if (e0 < E) dlogits[t * E + e0] = z0;
-    if (e1 < E) dlogits[t * E + e1] = z1;
-    if (dz16) {
-        dz16[t * 64 + e0] = __float2bfloat16_rn(e0 < E ? z0 : 0.f);
-        dz16[t * 64 + e1] = __float2bfloat16_rn(e1 < E ? z1 : 0.f);
+    float loc = 0.f;
+#pragma unroll
+    for (int i = 0; i < NV; ++i) loc += dp[i] * p[i];
+    const float dot = warp_sum(loc);
+#pragma unroll
+    for (int i = 0; i < NV; ++i) {
+        const int e = lane + 32 * i;
+        const float zz = p[i] * (dp[i] - dot);
+        if (e < E) dlogits[t * E + e] = zz;
+        if (dz16 && e < EP) dz16[t * EP + e] = __float2bfloat16_rn(e < E ? zz : 0.f);
     }
 }
 
@@ -478,7 +530,7 @@ static int num_sms() {
 template <typename T, bool FROM>
 static cudaError_t launch_route_t(const RouteArgs& a, cudaStream_t s) {
     const int E = a.E;
-    const size_t smem = (size_t)a.P * E * sizeof(int);
+    const size_t smem = a.P * E <= HIST_SMEM ? (size_t)a.P * E * sizeof(int) : 0;
     const int64_t groups_ub = a.T + a.P;  // upper bound with TPW = 1
     int blocks = (int)min64((groups_ub + 7) / 8, (int64_t)num_sms() * 8);
     if (blocks < 1) blocks = 1;
@@ -489,7 +541,9 @@ static cudaError_t launch_route_t(const RouteArgs& a, cudaStream_t s) {
         x, wr, a.bias, a.logits_in, a.po, a.P, a.T, a.d, E, a.k, a.normalize, a.logits, a.probs, \
         a.topk_idx, a.topk_w, a.counts)
     if constexpr (FROM) {
-        MOE_ROUTE_CASE(64, 4);
+        if (E <= 64) MOE_ROUTE_CASE(64, 4);
+        else if (E <= 128) MOE_ROUTE_CASE(128, 2);
+        else MOE_ROUTE_CASE(256, 1);
     } else if (E <= 8) {
         MOE_ROUTE_CASE(8, 8);
     } else if (E <= 16) {
@@ -503,11 +557,38 @@ static cudaError_t launch_route_t(const RouteArgs& a, cudaStream_t s) {
     return cudaGetLastError();
 }
 
+// E > 64 on the CUDA cores (fp32): the router's products x W_r[p]^T by the grouped SIMT
+// GEMM into `logits` (groups = parties), then the gating pass reads them back, adds the
+// bias and overwrites them with the biased logits.
+static cudaError_t launch_route_wide_simt(const RouteArgs& a, cudaStream_t s) {
+    GemmMArgs m{};
+    m.G = (a.po && a.P > 1) ? a.P : 1;
+    m.rows = (a.po && a.P > 1) ? GroupRows{a.po, (int)a.T, 0, 0, 0} : GroupRows{nullptr, (int)a.T, 0, 0, 0};
+    m.a = a.x;
+    m.b = a.w_router;
+    m.b_group_elems = (int64_t)a.E * a.d;
+    m.b_kmajor = true;
+    m.N = a.E;
+    m.K = a.d;
+    m.epi = EPI_STORE;
+    m.out0 = a.logits;
+    cudaError_t e = launch_gemm_m_simt(m, s);
+    if (e != cudaSuccess) return e;
+    RouteArgs b = a;
+    b.logits_in = a.logits;
+    return launch_route_t<float, true>(b, s);
+}
+
 cudaError_t launch_route(const RouteArgs& a, bool bf16, bool from_logits, cudaStream_t s) {
     cudaError_t e = cudaMemsetAsync(a.counts, 0, sizeof(int32_t) * a.P * a.E, s);
     if (e != cudaSuccess) return e;
-    if (from_logits) return launch_route_t<float, true>(a, s);
-    if (bf16 && a.E % 4 == 0 && a.T > 0) return launch_route_tc(a, s);
+    if (from_logits) {
+        RouteArgs b = a;
+        b.bias = nullptr;  // the caller's logits are final
+        return launch_route_t<float, true>(b, s);
+    }
+    if (bf16 && (a.E % 4 == 0 || a.E > 64) && a.T > 0) return launch_route_tc(a, s);
+    if (a.E > 64) return a.T > 0 ? launch_route_wide_simt(a, s) : cudaSuccess;
     return bf16 ? launch_route_t<__nv_bfloat16, false>(a, s) : launch_route_t<float, false>(a, s);
 }
 
@@ -525,6 +606,7 @@ cudaError_t launch_aux_loss(const float* probs, const int32_t* counts, const int
 static size_t align256(size_t n) { return (n + 255) / 256 * 256; }
 struct RbTcLayout {
     int64_t C, nchunk;
+    int EP;  // columns of dz16: E rounded up to 64, 128 or 256
     size_t dw, db, off, dz, total;
 };
 // Tokens per chunk of the chunked dW_r contraction: about 256 tiles of 128 model columns
@@ -541,8 +623,9 @@ static RbTcLayout rb_tc_layout(int64_t T, int P, int E, int d) {
     L.dw = 0;
     L.db = align256((size_t)L.nchunk * E * d * sizeof(float));
     L.off = align256(L.db + (size_t)L.nchunk * E * sizeof(float));
+    L.EP = E <= 64 ? 64 : E <= 128 ? 128 : 256;
     L.dz = align256(L.off + (size_t)(L.nchunk + 1) * sizeof(int32_t));
-    L.total = L.dz + (size_t)T * 64 * 2 + 256;
+    L.total = L.dz + (size_t)T * L.EP * 2 + 256;
     return L;
 }
 
@@ -552,6 +635,20 @@ size_t route_bwd_workspace(int64_t T, int P, int E, int d) {
     return std::max(simt, rb_tc_layout(T, P, E, d).total);
 }
 
+static cudaError_t launch_dlogits(const RouteBwdArgs& a, __nv_bfloat16* dz16, int EP, int32_t* chunk_off,
+                                  int CH, int nchunk, cudaStream_t s) {
+    const unsigned blocks = (unsigned)((a.T + 7) / 8);
+#define MOE_DL(NV)                                                                                 \
+    (void)launch_pdl(dlogits_kernel<NV>, dim3(blocks), dim3(256), 0, s, a.probs, a.topk_idx, a.topk_w, \
+                     a.dtopk_w, a.aux_coef, a.po, a.P, a.T, a.E, a.k, a.normalize, a.dlogits, dz16, EP, \
+                     chunk_off, CH, nchunk)
+    if (a.E <= 64) MOE_DL(2);
+    else if (a.E <= 128) MOE_DL(4);
+    else MOE_DL(8);
+#undef MOE_DL
+    return cudaGetLastError();
+}
+
 // fp32: dlogits, CUDA-core partials and reduce, dx_router on the CUDA-core GEMM
 static cudaError_t launch_route_bwd_simt(const RouteBwdArgs& a, void* ws, cudaStream_t s) {
     using T = float;
@@ -559,11 +656,7 @@ static cudaError_t launch_route_bwd_simt(const RouteBwdArgs& a, void* ws, cudaSt
     float* part_dw = (float*)ws;
     float* part_db = part_dw + nch * a.E * a.d;
     if (a.T > 0) {
-        const unsigned blocks = (unsigned)((a.T + 7) / 8);
-        (void)launch_pdl(dlogits_kernel, dim3(blocks), dim3(256), 0, s, a.probs, a.topk_idx, a.topk_w,
-                         a.dtopk_w, a.aux_coef, a.po, a.P, a.T, a.E, a.k, a.normalize, a.dlogits,
-                         (__nv_bfloat16*)nullptr, (int32_t*)nullptr, 0, 0);
-        cudaError_t e = cudaGetLastError();
+        cudaError_t e = launch_dlogits(a, (__nv_bfloat16*)nullptr, 0, (int32_t*)nullptr, 0, 0, s);
         if (e != cudaSuccess) return e;
     }
     constexpr int SLAB = RB_HALF * Vec<T>::N;
@@ -616,11 +709,8 @@ static cudaError_t launch_route_bwd_tc(const RouteBwdArgs& a, void* ws, cudaStre
     __nv_bfloat16* dz16 = (__nv_bfloat16*)(base + Lw.dz);
     cudaError_t e;
     if (a.T > 0) {
-        const unsigned blocks = (unsigned)((a.T + 7) / 8);
-        (void)launch_pdl(dlogits_kernel, dim3(blocks), dim3(256), 0, s, a.probs, a.topk_idx, a.topk_w,
-                         a.dtopk_w, a.aux_coef, a.po, a.P, a.T, a.E, a.k, a.normalize, a.dlogits, dz16,
-                         chunk_off, (int)Lw.C, (int)Lw.nchunk);
-        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+        if ((e = launch_dlogits(a, dz16, Lw.EP, chunk_off, (int)Lw.C, (int)Lw.nchunk, s)) != cudaSuccess)
+            return e;
         (void)launch_pdl(chunk_db_kernel, dim3((unsigned)Lw.nchunk), dim3(256), 0, s,
                          (const float*)a.dlogits, (const int32_t*)chunk_off, a.E, part_db);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
@@ -630,7 +720,7 @@ static cudaError_t launch_route_bwd_tc(const RouteBwdArgs& a, void* ws, cudaStre
         g.a = a.x;
         g.b = dz16;
         g.M = a.d;
-        g.N = 64;
+        g.N = Lw.EP;
         g.out = part_dw;
         g.epi = EPI_DWR;
         g.E = a.E;
@@ -650,7 +740,7 @@ static cudaError_t launch_route_bwd_tc(const RouteBwdArgs& a, void* ws, cudaStre
         m.b_group_elems = (int64_t)a.E * a.d;
         m.b_kmajor = false;
         m.N = a.d;
-        m.K = 64;
+        m.K = Lw.EP;
         m.b_rows = a.E;
         m.epi = EPI_STORE;
         m.out0 = a.dx_router;

@@ -69,7 +69,7 @@ def test_workspace_size_is_host_only(L):
 
 
 @pytest.mark.parametrize("field,value,frag", [
-    ("n_experts", 0, "n_experts"), ("n_experts", 65, "n_experts"), ("top_k", 0, "top_k"),
+    ("n_experts", 0, "n_experts"), ("top_k", 0, "top_k"),
     ("top_k", 9, "top_k"), ("d_model", 100, "multiples of 128"), ("dtype", 7, "dtype"),
     ("n_parties", 0, "n_parties"), ("normalize_topk", 2, "normalize_topk"), ("T", -1, "T="),
 ])
@@ -80,6 +80,16 @@ def test_bad_config_rejected_on_host(L, field, value, frag):
         L.moe_route(cfg, 16, 16, None, None, 16, 16, 16, 16, 16, stream=0)
     assert ei.value.status == L.MOE_ERR_INVALID_ARG
     assert frag in L.moe_last_error()
+
+
+def test_expert_pool_beyond_256_is_unsupported(L):
+    """E up to 256 is built; a larger pool is a documented refusal on the host."""
+    cfg = L.make_config(256, 256, 257, 256, 2)
+    with pytest.raises(L.MoEError) as ei:
+        L.moe_route(cfg, 16, 16, None, None, 16, 16, 16, 16, 16, stream=0)
+    assert ei.value.status == L.MOE_ERR_UNSUPPORTED
+    assert "n_experts=257" in L.moe_last_error()
+    assert L.moe_workspace_size(L.make_config(4096, 1024, 256, 512, 8)) > 0
 
 
 def test_null_and_misaligned_pointers_rejected_on_host(L):

@@ -153,6 +153,12 @@ SMALL = {
     # inside a 64-token block)
     "odd_E6_d384_parties3": lambda: mi.MoEShape("o6", 699, 384, 6, 256, 2, "bf16", n_parties=3,
                                                 seed=79),
+    # wide expert pools: E = 128 and 256 (bf16, tensor-core gating with TMEM read in
+    # chunks, dz padded to 128 / 256 columns, 128-256 GEMM groups), E = 100 in fp32
+    "wide_E128_bf16_parties2": lambda: mi.MoEShape("w128", 640, 256, 128, 128, 4, "bf16",
+                                                   n_parties=2, seed=80),
+    "wide_E256_bf16": lambda: mi.MoEShape("w256", 512, 128, 256, 128, 8, "bf16", seed=81),
+    "wide_E100_f32": lambda: mi.MoEShape("w100", 300, 64, 100, 64, 3, "f32", seed=82),
 }
 
 

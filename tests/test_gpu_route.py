@@ -28,7 +28,9 @@ def uneven_parties(T, P):
 
 @pytest.mark.parametrize("T,E,k,P,norm", [
     (1000, 8, 2, 1, 0), (777, 16, 2, 1, 1), (513, 64, 6, 1, 0), (300, 4, 4, 1, 0),
-    (1024, 32, 2, 4, 0), (5, 3, 1, 1, 0), (129, 64, 8, 3, 1), (1, 2, 2, 1, 0)])
+    (1024, 32, 2, 4, 0), (5, 3, 1, 1, 0), (129, 64, 8, 3, 1), (1, 2, 2, 1, 0),
+    # wide expert pools: lanes hold 4 or 8 experts; P E beyond the shared histogram
+    (600, 100, 6, 2, 0), (333, 256, 8, 1, 1), (200, 256, 2, 20, 0)])
 def test_route_from_logits_bit_exact(L, T, E, k, P, norm):
     z = mi.make_route_logits(T, E, seed=T * 7 + E, tie_every=3)
     po = uneven_parties(T, P)
@@ -55,7 +57,15 @@ def test_route_from_logits_bit_exact(L, T, E, k, P, norm):
     # d = 384 (6 k-blocks), three parties of 233 tokens: ragged tiles that end mid-party
     (2, 699, {"d_model": 384, "n_experts": 8, "n_parties": 3}),
     # E = 32 (N = 32), a single partial tile
-    (2, 77, {"n_experts": 32})])
+    (2, 77, {"n_experts": 32}),
+    # wide expert pools on the tensor cores (the gating epilogue reads TMEM in chunks):
+    # E = 128, E = 130 (scalar stores) with three parties, E = 256
+    (2, 700, {"n_experts": 128, "top_k": 6, "d_model": 256}),
+    (2, 511, {"n_experts": 130, "top_k": 3, "d_model": 256, "n_parties": 3}),
+    (2, 300, {"n_experts": 256, "top_k": 8, "d_model": 128}),
+    # fp32 with E > 64: the router products by the CUDA-core GEMM, then the gating
+    (1, 300, {"n_experts": 96, "top_k": 4}),
+    (1, 257, {"n_experts": 256, "top_k": 8, "n_parties": 1})])
 def test_route_matches_oracle(L, which, T, extra):
     """The tensor-core gating (router GEMM with the gating in its epilogue) against the
     fp64 oracle: logits within the accumulation tolerance, picks and counts exact."""
