@@ -61,7 +61,7 @@ def test_route_from_logits_bit_exact(L, T, E, k, P, norm):
     # wide expert pools on the tensor cores (the gating epilogue reads TMEM in chunks):
     # E = 128, E = 130 (scalar stores) with three parties, E = 256
     (2, 700, {"n_experts": 128, "top_k": 6, "d_model": 256}),
-    (2, 511, {"n_experts": 130, "top_k": 3, "d_model": 256, "n_parties": 3}),
+    (2, 513, {"n_experts": 130, "top_k": 3, "d_model": 256, "n_parties": 3}),
     (2, 300, {"n_experts": 256, "top_k": 8, "d_model": 128}),
     # fp32 with E > 64: the router products by the CUDA-core GEMM, then the gating
     (1, 300, {"n_experts": 96, "top_k": 4}),
