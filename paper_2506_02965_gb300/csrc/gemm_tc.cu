@@ -54,6 +54,10 @@ struct Params {
     // EPI_ROUTE: out0 = logits, out1 = probs (fp32 [T,E]), aux = bias [P,E] or null
     int E, k, normalize, hist_n;
     int band;  // tile order: bands of `band` M-tiles, each swept along N (set at launch)
+    // operand bytes for the per-group choice of the tile order: the bytes of one A row
+    // (M-variable: K elements; K-variable: Mout elements per contraction row), of one B
+    // contraction row (K-variable), and of all of B (M-variable: one group's weights)
+    int64_t a_row_bytes, b_row_bytes, b_all_bytes;
     int32_t* topk_idx;
     float* topk_w;
     int32_t* counts;
@@ -596,7 +600,18 @@ __global__ void __launch_bounds__(THREADS, 1)
     // of the persistent grid, C of them) then cover about band x C/band output tiles and
     // read band A blocks and C/band B blocks, instead of one A block and C B blocks when
     // whole rows of N-tiles come first (band ~ sqrt(C) minimises the blocks per round;
-    // the A blocks of a band also stay in L2 while it sweeps N).
+    // the A blocks of a band also stay in L2 while it sweeps N). When all of a group's B
+    // fits in L2, whole rows of N-tiles first (band 1) read it from DRAM once and each A
+    // block once; else when all of its A fits, whole columns of M-tiles first (band =
+    // the group's M-tiles) do the same with A resident.
+    constexpr int64_t kL2Resident = 48ll << 20;  // bytes of an operand kept in L2
+    auto group_band = [&](const Params& q, int64_t rows_g, int mt_g) -> int {
+        const int64_t a_all = (int64_t)rows_g * q.a_row_bytes;
+        const int64_t b_all = q.b_row_bytes ? (int64_t)rows_g * q.b_row_bytes : q.b_all_bytes;
+        if (b_all > 0 && b_all <= kL2Resident) return 1;
+        if (a_all > 0 && a_all <= kL2Resident) return mt_g;
+        return q.band;
+    };
     auto band_split = [&](int local, int mt_g, int nt_g, int band, int* mt, int* nt) {
         const int gmx = band > 0 ? band : 1;
         const int b = local / (gmx * nt_g);
@@ -615,7 +630,8 @@ __global__ void __launch_bounds__(THREADS, 1)
                 const int g = s_order[(t - s_total1) / per], l2 = (t - s_total1) % per;
                 const int tn2 = p2.N / BN;
                 int mt2, nt2;
-                band_split(l2, p2.Mout / BM, tn2, p2.band, &mt2, &nt2);
+                band_split(l2, p2.Mout / BM, tn2,
+                           group_band(p2, p2.offsets[g + 1] - p2.offsets[g], p2.Mout / BM), &mt2, &nt2);
                 ti.dw = true;
                 ti.g = g;
                 ti.we = p2.gexp ? p2.gexp[g] : g;
@@ -641,8 +657,10 @@ __global__ void __launch_bounds__(THREADS, 1)
         const int g = lo;
         const int local = t - s_tile_start[g];
         const int g_end = (g + 1 < p.G) ? s_tile_start[g + 1] : s_total1;
+        const int mt_g = (g_end - s_tile_start[g]) / tiles_n;
+        const int64_t rows_g = p.offsets ? (int64_t)(p.offsets[g + 1] - p.offsets[g]) : (int64_t)p.rows;
         int mt, nt;
-        band_split(local, (g_end - s_tile_start[g]) / tiles_n, tiles_n, p.band, &mt, &nt);
+        band_split(local, mt_g, tiles_n, group_band(p, rows_g, mt_g), &mt, &nt);
         ti.g = g;
         ti.we = p.gexp ? p.gexp[g] : g;
         ti.m0 = mt * BMP + (int)rank * BM;
@@ -1443,6 +1461,8 @@ cudaError_t launch_gemm_m(const GemmMArgs& g, bool bf16, cudaStream_t s) {
     p.aux = g.aux;
     p.wait_ns = g_wait_ns;
     p.gexp = g.group_expert;
+    p.a_row_bytes = (int64_t)g.K * 2;
+    p.b_all_bytes = (int64_t)g.N * (g.b_kmajor ? g.K : (g.b_rows ? g.b_rows : g.K)) * 2;
     // A rows in the 2D view: OFFSETS -> all routed rows; UNIFORM -> groups * stride (or rows)
     const int64_t a_rows = g.rows.offsets ? (int64_t)g.rows.rows
                                           : std::max<int64_t>(g.rows.rows, (int64_t)(g.G - 1) * g.rows.a_stride + g.rows.rows);
@@ -1518,6 +1538,8 @@ cudaError_t launch_gemm_k(const GemmKArgs& g, bool bf16, cudaStream_t s) {
     p.out0 = g.out;
     p.wait_ns = g_wait_ns;
     p.gexp = g.group_expert;
+    p.a_row_bytes = (int64_t)g.M * 2;
+    p.b_row_bytes = (int64_t)g.N * 2;
     const int64_t rows_a = g.rows.offsets ? (int64_t)g.rows.rows
                                           : std::max<int64_t>(g.rows.rows, (int64_t)(g.G - 1) * g.rows.a_stride + g.rows.rows);
     const int64_t rows_b = g.rows.offsets ? (int64_t)g.rows.rows
@@ -1566,6 +1588,8 @@ cudaError_t launch_gemm_mk(const GemmMArgs& g, const GemmKArgs& k, cudaStream_t 
     p.wait_ns = g_wait_ns;
     p.gexp = g.group_expert;
     p.b_group_rows = g.b_rows ? g.b_rows : g.K;
+    p.a_row_bytes = (int64_t)g.K * 2;
+    p.b_all_bytes = (int64_t)g.N * p.b_group_rows * 2;
     const int64_t a_rows = (int64_t)g.rows.rows, o_rows = a_rows;
     CUtensorMap ma, mb, mo0, mo1;
     if (!make_map(&ma, g.a, g.K, a_rows, BM)) return cudaErrorInvalidValue;
@@ -1587,6 +1611,8 @@ cudaError_t launch_gemm_mk(const GemmMArgs& g, const GemmKArgs& k, cudaStream_t 
     p2.out0 = k.out;
     p2.wait_ns = g_wait_ns;
     p2.gexp = k.group_expert;
+    p2.a_row_bytes = (int64_t)k.M * 2;
+    p2.b_row_bytes = (int64_t)k.N * 2;
     CUtensorMap ma2, mb2, mo2;
     if (!make_map(&ma2, k.a, k.M, (int64_t)k.rows.rows, 64)) return cudaErrorInvalidValue;
     if (!make_map(&mb2, k.b, k.N, (int64_t)k.rows.rows, 64)) return cudaErrorInvalidValue;
