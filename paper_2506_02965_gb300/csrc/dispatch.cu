@@ -164,33 +164,43 @@ __global__ void __launch_bounds__(DCH) slot_kernel(const int32_t* __restrict__ i
     }
 }
 
-// x_perm[r] = x[token_of[r]]: one warp per permuted row, 16-byte vectors.
+// x_perm[slot_of[t,j]] = x[t] for every pick j: one warp per token reads its row once
+// (16-byte vectors, U of them in flight per lane) and writes it to its k rows of x_perm.
+// A slot outside [0, T k) is skipped and recorded as MOE_ERR_DEVICE_CHECK.
 template <typename T>
 __global__ void __launch_bounds__(256) gather_kernel(const T* __restrict__ x,
-                                                     const int32_t* __restrict__ token_of,
-                                                     int64_t TK, int64_t Tn, int d, T* x_perm) {
+                                                     const int32_t* __restrict__ slot_of,
+                                                     int64_t Tn, int d, int k, T* x_perm) {
     pdl_begin();
     const int lane = threadIdx.x & 31;
-    const int64_t r = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-    if (r >= TK) return;
-    const int64_t t = token_of[r];
-    if (t < 0 || t >= Tn) {
-        if (lane == 0) record_status(MOE_ERR_DEVICE_CHECK);
-        return;
+    const int64_t t = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    if (t >= Tn) return;
+    int32_t slot[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+        slot[j] = j < k ? slot_of[t * k + j] : -1;
+        if (j < k && (slot[j] < 0 || (int64_t)slot[j] >= Tn * k)) {
+            if (lane == 0) record_status(MOE_ERR_DEVICE_CHECK);
+            slot[j] = -1;
+        }
     }
     constexpr int VN = Vec<T>::N;
     constexpr int U = 4;  // vectors per lane in flight
     const int nv = d / VN;
     const T* src = x + t * d;
-    T* dst = x_perm + r * d;
     for (int v0 = lane; v0 < nv; v0 += 32 * U) {
         uint4 buf[U];
 #pragma unroll
         for (int u = 0; u < U; ++u)
             if (v0 + 32 * u < nv) buf[u] = Vec<T>::raw_load(src + (v0 + 32 * u) * VN);
 #pragma unroll
-        for (int u = 0; u < U; ++u)
-            if (v0 + 32 * u < nv) Vec<T>::raw_store(dst + (v0 + 32 * u) * VN, buf[u]);
+        for (int j = 0; j < 8; ++j) {
+            if (slot[j] < 0) continue;
+            T* dst = x_perm + (int64_t)slot[j] * d;
+#pragma unroll
+            for (int u = 0; u < U; ++u)
+                if (v0 + 32 * u < nv) Vec<T>::raw_store(dst + (v0 + 32 * u) * VN, buf[u]);
+        }
     }
 }
 
@@ -395,6 +405,18 @@ __global__ void __launch_bounds__(256, 3) unpermute_reduce_kernel(
 }
 
 // ----------------------------------------------------------------------------- launchers
+static cudaError_t launch_gather(const void* x, const int32_t* slot_of, int64_t T, int d, int k, bool bf16,
+                                 void* x_perm, cudaStream_t s) {
+    const unsigned blocks = (unsigned)((T + 7) / 8);
+    if (bf16)
+        (void)launch_pdl(gather_kernel<__nv_bfloat16>, dim3(blocks), dim3(256), 0, s, (const __nv_bfloat16*)x,
+                         slot_of, T, d, k, (__nv_bfloat16*)x_perm);
+    else
+        (void)launch_pdl(gather_kernel<float>, dim3(blocks), dim3(256), 0, s, (const float*)x, slot_of, T, d, k,
+                         (float*)x_perm);
+    return cudaGetLastError();
+}
+
 size_t dispatch_workspace(int64_t T, int E) {
     const int64_t nch = (T + DCH - 1) / DCH;
     return (size_t)nch * E * sizeof(int32_t) + 256;
@@ -421,16 +443,8 @@ cudaError_t launch_dispatch(const int32_t* topk_idx, const void* x, int64_t T, i
                      slot_of, token_of, owner ? P : 1, group_expert);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    const int64_t TK = T * k;
-    if (TK == 0) return cudaSuccess;
-    const unsigned blocks = (unsigned)((TK + 7) / 8);
-    if (bf16)
-        (void)launch_pdl(gather_kernel<__nv_bfloat16>, dim3(blocks), dim3(256), 0, s, (const __nv_bfloat16*)x, token_of, TK, T,
-                                                            d, (__nv_bfloat16*)x_perm);
-    else
-        (void)launch_pdl(gather_kernel<float>, dim3(blocks), dim3(256), 0, s, (const float*)x, token_of, TK, T, d,
-                                                    (float*)x_perm);
-    return cudaGetLastError();
+    if (T * k == 0) return cudaSuccess;
+    return launch_gather(x, slot_of, T, d, k, bf16, x_perm, s);
 }
 
 cudaError_t launch_combine_fwd(const void* y_perm, const float* topk_w, const int32_t* slot_of,
@@ -542,15 +556,7 @@ cudaError_t launch_dispatch_noalloc(const int32_t* topk_idx, const void* x, int6
                      slot_of, token_of, 1, (int32_t*)nullptr);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    const int64_t TK = T * k;
-    const unsigned blocks = (unsigned)((TK + 7) / 8);
-    if (bf16)
-        (void)launch_pdl(gather_kernel<__nv_bfloat16>, dim3(blocks), dim3(256), 0, s, (const __nv_bfloat16*)x, token_of, TK, T,
-                                                            d, (__nv_bfloat16*)x_perm);
-    else
-        (void)launch_pdl(gather_kernel<float>, dim3(blocks), dim3(256), 0, s, (const float*)x, token_of, TK, T, d,
-                                                    (float*)x_perm);
-    return cudaGetLastError();
+    return launch_gather(x, slot_of, T, d, k, bf16, x_perm, s);
 }
 
 cudaError_t dispatch_status(cudaStream_t s, int* code) { return tu_status_read_clear(s, code); }

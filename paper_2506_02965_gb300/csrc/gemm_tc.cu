@@ -23,6 +23,10 @@ namespace tc {
 
 constexpr int BM = 128;
 constexpr int BK = 64;  // 64 bf16 = 128 bytes = one 128B-swizzle row
+// Contraction rows per k-block: BK, except for CTA-pair K-variable tiles (weight
+// gradients), whose operands are both MN-major (64-element TMA boxes): 128-row boxes
+// there halve the boxes and stage hand-offs per byte (3 stages of 64 KiB per CTA).
+__host__ __device__ constexpr int kblock_rows(bool var_k, bool pair) { return (var_k && pair) ? 128 : BK; }
 constexpr int STAGES = 4;
 constexpr int EPI_WARPS = 4;
 constexpr int THREADS = 64 + 32 * EPI_WARPS;  // TMA warp, MMA warp, epilogue warps
@@ -532,8 +536,10 @@ __global__ void __launch_bounds__(THREADS, 1)
     constexpr int NPAIR = PAIR ? 2 : 1;
     constexpr int BNL = BN / NPAIR;  // B rows held by this CTA
     constexpr int BMP = BM * NPAIR;  // rows of one (pair) tile
-    constexpr uint32_t A_BYTES = BM * BK * 2;
-    constexpr uint32_t B_BYTES = BNL * BK * 2;
+    constexpr int KB = kblock_rows(VAR_K, PAIR);  // contraction rows per k-block
+    constexpr uint32_t ATOM = KB * 128;              // bytes of one 64-wide MN-major box
+    constexpr uint32_t A_BYTES = BM * KB * 2;
+    constexpr uint32_t B_BYTES = BNL * KB * 2;
     constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
     constexpr int NST = num_stages(STAGE_BYTES, EPI);
     constexpr uint32_t IDESC = instr_desc<BN, A_MN, B_MN, BMP>();
@@ -681,8 +687,8 @@ __global__ void __launch_bounds__(THREADS, 1)
             ti.a_row = a0;
             ti.b_row = b0;
             ti.out_row = 0;
-            ti.k_iters = (int)((nrows + BK - 1) / BK);
-            ti.last_rows = (int)(nrows - (int64_t)(ti.k_iters - 1) * BK);
+            ti.k_iters = (int)((nrows + KB - 1) / KB);
+            ti.last_rows = (int)(nrows - (int64_t)(ti.k_iters - 1) * KB);
         } else {
             ti.mvalid = (int)nrows;
             ti.a_row = a0;
@@ -797,7 +803,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                     // K-variable pair, peer, partial last k-block: its copies land on its own
                     // barrier; the MMA warp zeroes the rows past the group's end and then
                     // credits these bytes to the leader's full barrier
-                    const bool part_peer = PAIR && VAR_K && rank == 1 && kb == ti.k_iters - 1 && ti.last_rows < BK;
+                    const bool part_peer = PAIR && VAR_K && rank == 1 && kb == ti.k_iters - 1 && ti.last_rows < KB;
                     const uint32_t fb = part_peer ? pfull_bar(stage)
                                                   : (PAIR ? map_to_rank(full_bar(stage), 0) : full_bar(stage));
                     local_bar = part_peer;
@@ -816,7 +822,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                     } else {
                         mbar_expect_tx(fb, STAGE_BYTES);
                     }
-                    const int k0 = kb * BK;
+                    const int k0 = kb * KB;
                     const bool dw = DW2 && ti.dw;
                     if (!A_MN && !dw) {
                         load(sa, &tmA, fb, k0, (int)(ti.a_row + ti.m0));
@@ -824,7 +830,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                         const CUtensorMap* mA = dw ? &tmA2 : &tmA;
 #pragma unroll
                         for (int i = 0; i < BM / 64; ++i)
-                            load(sa + i * 8192, mA, fb, ti.m0 + 64 * i, (int)(ti.a_row + k0));
+                            load(sa + i * ATOM, mA, fb, ti.m0 + 64 * i, (int)(ti.a_row + k0));
                     }
                     if (EPI == EPI_SWIGLU_FWD) {
                         // 128 gate rows then 128 up rows of the same features; in a pair the
@@ -843,7 +849,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                         const CUtensorMap* mB = dw ? &tmB2 : &tmB;
 #pragma unroll
                         for (int i = 0; i < BNL / 64; ++i)
-                            load(sb + i * 8192, mB, fb, ti.n0 + (int)rank * BNL + 64 * i, (int)krow);
+                            load(sb + i * ATOM, mB, fb, ti.n0 + (int)rank * BNL + 64 * i, (int)krow);
                     }
                     issued_phase[stage] = (int)phase;
                     if (++stage == NST) {
@@ -905,9 +911,9 @@ __global__ void __launch_bounds__(THREADS, 1)
                 // group. Only K=16 steps that contain valid rows are issued, and inside the
                 // last of them the A rows past the group's end are zeroed (A alone suffices:
                 // their products with any finite B row vanish).
-                int ksteps = BK / 16;
+                int ksteps = KB / 16;
                 const bool dwt = DW2 && ti.dw;
-                if ((VAR_K || dwt) && kb == ti.k_iters - 1 && ti.last_rows < BK) {
+                if ((VAR_K || dwt) && kb == ti.k_iters - 1 && ti.last_rows < KB) {
                     ksteps = (ti.last_rows + 15) / 16;
                     const int zr0 = ti.last_rows, zr1 = ksteps * 16;
                     if (zr1 > zr0) {
@@ -915,7 +921,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                         const int per_box = (zr1 - zr0) * 8;  // 16-byte words
 #pragma unroll
                         for (int b = 0; b < BM / 64; ++b) {
-                            uint4* z = reinterpret_cast<uint4*>(base + b * 8192 + zr0 * 128);
+                            uint4* z = reinterpret_cast<uint4*>(base + b * ATOM + zr0 * 128);
                             for (int i = lane; i < per_box; i += 32) z[i] = make_uint4(0, 0, 0, 0);
                         }
                         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -925,13 +931,13 @@ __global__ void __launch_bounds__(THREADS, 1)
                 fence_after();
                 if (lane == 0) {
 #pragma unroll
-                    for (int kk = 0; kk < BK / 16; ++kk) {
+                    for (int kk = 0; kk < KB / 16; ++kk) {
                         if (kk >= ksteps) break;
                         uint64_t ad, bd;
                         if (!A_MN && !dwt) ad = smem_desc(sa + kk * 32, 16, 1024);
-                        else ad = smem_desc(sa + kk * 2048, 8192, 1024);
+                        else ad = smem_desc(sa + kk * 2048, ATOM, 1024);
                         if (!B_MN) bd = smem_desc(sb + kk * 32, 16, 1024);
-                        else bd = smem_desc(sb + kk * 2048, 8192, 1024);
+                        else bd = smem_desc(sb + kk * 2048, ATOM, 1024);
                         if constexpr (PAIR) mma_bf16_pair(tmem_d, ad, bd, IDESC, (kb | kk) ? 1u : 0u);
                         else mma_bf16(tmem_d, ad, bd, dwt ? IDESC_DW : IDESC, (kb | kk) ? 1u : 0u);
                     }
@@ -981,7 +987,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                 for (int t = tile0; t < total_tiles && ok2; t += tile_step) {
                     const Tile ti = tile_at(t);
                     for (int kb = 0; kb < ti.k_iters; ++kb) {
-                        if (kb == ti.k_iters - 1 && ti.last_rows < BK) {
+                        if (kb == ti.k_iters - 1 && ti.last_rows < KB) {
                             if (!mbar_wait(pfull_bar(st2), (wpar >> st2) & 1u, abort_flag, p.wait_ns)) {
                                 ok2 = false;
                                 break;
@@ -993,7 +999,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                                 const int per_box = (zr1 - zr0) * 8;  // 16-byte words
 #pragma unroll
                                 for (int b = 0; b < BM / 64; ++b) {
-                                    uint4* z = reinterpret_cast<uint4*>(base + b * 8192 + zr0 * 128);
+                                    uint4* z = reinterpret_cast<uint4*>(base + b * ATOM + zr0 * 128);
                                     for (int i = lane; i < per_box; i += 32) z[i] = make_uint4(0, 0, 0, 0);
                                 }
                                 asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -1344,11 +1350,13 @@ static cudaError_t launch(const CUtensorMap& ma, const CUtensorMap& mb, const CU
     Params P1 = p;
     Params P2 = p2 ? *p2 : p;
     constexpr int NPAIR = PAIR ? 2 : 1;
-    constexpr int NST = num_stages((uint32_t)(BM * BK * 2 + BN / NPAIR * BK * 2), EPI);
+    constexpr int KB = kblock_rows(VAR_K, PAIR);
+    constexpr int STB = BM * KB * 2 + BN / NPAIR * KB * 2;  // bytes of one operand stage
+    constexpr int NST = num_stages((uint32_t)STB, EPI);
     const int extra_max = EPI == EPI_ROUTE ? 64 * 64 * 4 : EPI_WARPS * epi_stage_bytes(EPI);
     const int extra = EPI == EPI_ROUTE ? p.hist_n * 4 : EPI_WARPS * epi_stage_bytes(EPI);
-    const int smem_max = NST * (BM * BK * 2 + BN / NPAIR * BK * 2) + 1024 + extra_max;
-    const int smem = NST * (BM * BK * 2 + BN / NPAIR * BK * 2) + 1024 + extra;
+    const int smem_max = NST * STB + 1024 + extra_max;
+    const int smem = NST * STB + 1024 + extra;
     static bool attr_set = false;
     if (!attr_set) {
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_max);
@@ -1545,8 +1553,10 @@ cudaError_t launch_gemm_k(const GemmKArgs& g, bool bf16, cudaStream_t s) {
     const int64_t rows_b = g.rows.offsets ? (int64_t)g.rows.rows
                                           : std::max<int64_t>(g.rows.rows, (int64_t)(g.G - 1) * g.rows.b_stride + g.rows.rows);
     CUtensorMap ma, mb, mo;
-    if (!make_map(&ma, g.a, g.M, rows_a, 64)) return cudaErrorInvalidValue;
-    if (!make_map(&mb, g.b, g.N, rows_b, 64)) return cudaErrorInvalidValue;
+    const bool pair = g.epi == EPI_STORE && gemm_k_uses_pairs(g);
+    const int kbr = kblock_rows(true, pair);  // box rows of the MN-major operands
+    if (!make_map(&ma, g.a, g.M, rows_a, kbr)) return cudaErrorInvalidValue;
+    if (!make_map(&mb, g.b, g.N, rows_b, kbr)) return cudaErrorInvalidValue;
     const int64_t tiles = (int64_t)g.G * (g.M / BM);
     if (g.epi == EPI_DWR) {  // fp32 partials, N = 64, 128 or 256 (experts, zero-padded)
         if ((g.N != 64 && g.N != 128 && g.N != 256) || g.M % BM) return cudaErrorInvalidValue;
@@ -1556,7 +1566,7 @@ cudaError_t launch_gemm_k(const GemmKArgs& g, bool bf16, cudaStream_t s) {
         return launch<256, true, true, EPI_DWR>(ma, mb, ma, ma, p, tiles, s);
     }
     if (!make_map(&mo, g.out, g.N, (int64_t)g.G * g.M, 0, true)) return cudaErrorInvalidValue;
-    if (gemm_k_uses_pairs(g))
+    if (pair)
         return launch<256, true, true, EPI_STORE, true>(ma, mb, mo, mo, p, (int64_t)g.G * (g.M / 256) * (g.N / 256), s);
     if (g.N % 256 == 0) return launch<256, true, true, EPI_STORE>(ma, mb, mo, mo, p, tiles * (g.N / 256), s);
     return launch<128, true, true, EPI_STORE>(ma, mb, mo, mo, p, tiles * (g.N / 128), s);

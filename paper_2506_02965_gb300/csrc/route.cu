@@ -218,11 +218,20 @@ __global__ void __launch_bounds__(256) route_kernel(
 
 // ----------------------------------------------------------------------------- aux loss
 // One 8-CTA thread-block cluster per party: each CTA sums probs[t, e] over its slice
-// of the party's tokens (fixed order inside the CTA), then CTA 0 of the cluster adds
-// the 8 partial rows from distributed shared memory in rank order. Deterministic,
-// no workspace, no floating-point atomics.
+// of the party's tokens, then CTA 0 of the cluster adds the 8 partial rows from
+// distributed shared memory in rank order. Inside a CTA, thread (s, e) of S = 2^j
+// stripes per expert loads AUX_U values of its stripe at once (independent loads in
+// flight) and adds them in order; the stripes are then added by a fixed binary tree.
+// Deterministic, no workspace, no floating-point atomics.
 constexpr int AUX_CLUSTER = 8;
 constexpr int AUX_THREADS = 1024;
+constexpr int AUX_U = 8;
+
+__device__ __forceinline__ int pow2_floor(int v) {
+    int r = 1;
+    while (2 * r <= v) r *= 2;
+    return r;
+}
 
 __global__ void __cluster_dims__(AUX_CLUSTER, 1, 1) __launch_bounds__(AUX_THREADS)
     aux_loss_kernel(const float* __restrict__ probs, const int32_t* __restrict__ counts,
@@ -239,26 +248,28 @@ __global__ void __cluster_dims__(AUX_CLUSTER, 1, 1) __launch_bounds__(AUX_THREAD
     const int64_t per = (n + AUX_CLUSTER - 1) / AUX_CLUSTER;
     const int64_t lo = a + min64(n, per * rank), hi = a + min64(n, per * (rank + 1));
     const int tid = threadIdx.x;
-    const int stripes = AUX_THREADS / E;
-    float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+    const int stripes = pow2_floor(AUX_THREADS / E);
+    float acc = 0.f;
     if (tid < stripes * E) {
         const int e = tid % E, st = tid / E;
-        int64_t t = lo + st;
-        for (; t + 3 * stripes < hi; t += 4 * stripes) {
-            s0 += probs[t * E + e];
-            s1 += probs[(t + stripes) * E + e];
-            s2 += probs[(t + 2 * stripes) * E + e];
-            s3 += probs[(t + 3 * stripes) * E + e];
+        for (int64_t t = lo + st; t < hi; t += (int64_t)AUX_U * stripes) {
+            float v[AUX_U];
+#pragma unroll
+            for (int u = 0; u < AUX_U; ++u) {
+                const int64_t tt = t + (int64_t)u * stripes;
+                v[u] = tt < hi ? probs[tt * E + e] : 0.f;
+            }
+#pragma unroll
+            for (int u = 0; u < AUX_U; ++u) acc += v[u];
         }
-        for (; t < hi; t += stripes) s0 += probs[t * E + e];
     }
-    s_part[tid] = (s0 + s1) + (s2 + s3);
+    s_part[tid] = acc;
     __syncthreads();
-    if (tid < E) {
-        float tot = 0.f;
-        for (int st = 0; st < stripes; ++st) tot += s_part[st * E + tid];
-        s_col[tid] = tot;
+    for (int h = stripes / 2; h > 0; h >>= 1) {
+        if (tid < h * E) s_part[tid] += s_part[tid + h * E];
+        __syncthreads();
     }
+    if (tid < E) s_col[tid] = s_part[tid];
     cluster.sync();
     if (rank == 0 && tid < E) {
         float tot = 0.f;
@@ -359,25 +370,39 @@ __global__ void __launch_bounds__(256) dlogits_kernel(
 }
 
 // dbias partial of one token chunk: part_db[c][e] = sum of dlogits[t][e] over the chunk.
-// Thread (g, e) of a block, g < G = 256 / E token groups, sums tokens g, g + G, ...; the
-// groups are then added in order (fixed order: deterministic).
-__global__ void __launch_bounds__(256) chunk_db_kernel(const float* __restrict__ dz,
-                                                      const int32_t* __restrict__ chunk_off, int E,
-                                                      float* part_db) {
+// Thread (g, e) of a block, g < G = 2^j <= 1024 / E token groups, loads CDB_U tokens
+// g, g + G, ... at once and adds them in order; the groups are then added by a fixed
+// binary tree (deterministic).
+constexpr int CDB_THREADS = 1024;
+constexpr int CDB_U = 8;
+__global__ void __launch_bounds__(CDB_THREADS) chunk_db_kernel(const float* __restrict__ dz,
+                                                              const int32_t* __restrict__ chunk_off, int E,
+                                                              float* part_db) {
     pdl_begin();
-    __shared__ float s_part[256];
-    const int c = blockIdx.x, G = 256 / E, e = threadIdx.x % E, g = threadIdx.x / E;
+    __shared__ float s_part[CDB_THREADS];
+    const int c = blockIdx.x, G = pow2_floor(CDB_THREADS / E);
+    const int e = threadIdx.x % E, g = threadIdx.x / E;
     const int64_t a = chunk_off[c], b = chunk_off[c + 1];
     float acc = 0.f;
-    if (g < G)
-        for (int64_t t = a + g; t < b; t += G) acc += dz[t * E + e];
-    s_part[threadIdx.x] = acc;
-    __syncthreads();
-    if (threadIdx.x < E) {
-        float sum = 0.f;
-        for (int q = 0; q < G; ++q) sum += s_part[q * E + threadIdx.x];
-        part_db[(int64_t)c * E + threadIdx.x] = sum;
+    if (g < G) {
+        for (int64_t t = a + g; t < b; t += (int64_t)CDB_U * G) {
+            float v[CDB_U];
+#pragma unroll
+            for (int u = 0; u < CDB_U; ++u) {
+                const int64_t tt = t + (int64_t)u * G;
+                v[u] = tt < b ? dz[tt * E + e] : 0.f;
+            }
+#pragma unroll
+            for (int u = 0; u < CDB_U; ++u) acc += v[u];
+        }
     }
+    s_part[threadIdx.x] = (g < G) ? acc : 0.f;
+    __syncthreads();
+    for (int h = G / 2; h > 0; h >>= 1) {
+        if (threadIdx.x < h * E) s_part[threadIdx.x] += s_part[threadIdx.x + h * E];
+        __syncthreads();
+    }
+    if (threadIdx.x < E) part_db[(int64_t)c * E + threadIdx.x] = s_part[threadIdx.x];
 }
 
 // Partial dW_r = dlogits^T x and db over one chunk of RB_CH tokens of one party, for
@@ -711,7 +736,7 @@ static cudaError_t launch_route_bwd_tc(const RouteBwdArgs& a, void* ws, cudaStre
     if (a.T > 0) {
         if ((e = launch_dlogits(a, dz16, Lw.EP, chunk_off, (int)Lw.C, (int)Lw.nchunk, s)) != cudaSuccess)
             return e;
-        (void)launch_pdl(chunk_db_kernel, dim3((unsigned)Lw.nchunk), dim3(256), 0, s,
+        (void)launch_pdl(chunk_db_kernel, dim3((unsigned)Lw.nchunk), dim3(CDB_THREADS), 0, s,
                          (const float*)a.dlogits, (const int32_t*)chunk_off, a.E, part_db);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
         GemmKArgs g{};

@@ -39,8 +39,9 @@ def picks(T, E, k, pattern, seed=0):
     raise ValueError(pattern)
 
 
-# rows per expert around the K=16 MMA step and the 64-row k-block (empty, one row, ...)
-EDGE_SIZES = [0, 1, 15, 16, 17, 63, 64, 65, 128, 200]
+# rows per expert around the K=16 MMA step and the 64- and 128-row k-blocks (empty, one
+# row, ...)
+EDGE_SIZES = [0, 1, 15, 16, 17, 63, 64, 65, 127, 128, 129, 200, 255, 256, 257]
 
 
 CASES = [(1000, 8, 2, "uniform", "bf16"), (333, 16, 2, "skewed", "bf16"),

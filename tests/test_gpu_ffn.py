@@ -151,9 +151,10 @@ def test_expert_ffn_single_cta_and_pair_tiles(L, pairs):
         for case in [(777, 512, 8, 512, 2, "skewed", "bf16", 0, 0),
                      (300, 256, 4, 256, 2, "uniform", "bf16", 1, 256),
                      (1024, 1024, 16, 2816, 2, "uniform", "bf16", 0, 0),
-                     # experts of 0, 1, 15, 16, 17, 63, 64, 65, 128, 200 rows: every way the
-                     # weight gradients' last k-block can end (pairs: zeroed on both CTAs)
-                     (569, 256, 10, 256, 1, "edges", "bf16", 0, 0)]:
+                     # experts of 0, 1, 15, 16, 17, 63, 64, 65, 127, 128, 129, 200, 255, 256,
+                     # 257 rows: every way the weight gradients' last k-block (64 rows, 128 for
+                     # pair tiles) can end (pairs: zeroed on both CTAs)
+                     (1593, 256, 15, 256, 1, "edges", "bf16", 0, 0)]:
             test_expert_ffn_fwd_bwd(L, case)
     finally:
         L.moe_set_gemm_pairs(2)
