@@ -1052,10 +1052,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         if constexpr (EPI == EPI_SWIGLU_BWD) {
             if (tile0 < total_tiles) {
                 const Tile tf = tile_at(tile0);
-                if (!(DW2 && tf.dw)) {  // the first tile's first two chunks, before its mainloop ends
-                    gu_issue(tf, 0);
-                    gu_issue(tf, 1);
-                }
+                if (!(DW2 && tf.dw)) gu_issue(tf, 0);
             }
         }
         for (int t = tile0; t < total_tiles; t += tile_step) {
@@ -1113,69 +1110,59 @@ __global__ void __launch_bounds__(THREADS, 1)
                 }
             } else if constexpr (EPI == EPI_SWIGLU_BWD) {
                 // dA in TMEM. G and U of each 32-column chunk arrive by TMA in one of two
-                // staging buffers, two chunks ahead of their use: once a chunk's G and U
-                // are read, its buffer takes the load of the chunk two further on (this
-                // tile's, or the next tile's first ones). dG and dU go straight from the
-                // registers to global memory (each lane its row), so a buffer never waits
-                // for a store to leave it.
+                // staging buffers (the next chunk's load is in flight while this one is
+                // computed); dG and dU overwrite them in place and leave by TMA store.
                 const int F = p.F;
                 __nv_bfloat16* dh = (__nv_bfloat16*)p.out0 + (ti.out_row + m) * (int64_t)(2 * F) + ti.n0;
                 constexpr int NCH = BN / 32;
-                // the chunk `a` places after chunk c of this tile (at most one tile ahead)
-                auto ahead = [&](int c, int a, Tile* tn, int* cn) -> bool {
-                    const int c2 = c + a;
-                    if (c2 < NCH) {
-                        *tn = ti;
-                        *cn = c2;
-                        return true;
-                    }
-                    if (t + tile_step >= total_tiles) return false;
-                    const Tile nx = tile_at(t + tile_step);
-                    if (DW2 && nx.dw) return false;
-                    *tn = nx;
-                    *cn = c2 - NCH;
-                    return true;
-                };
-                // this tile's first two chunks, where the previous tile did not issue them
-                // (the first tile of the warp)
-                while ((int)(gu_issued - gu_chunk) < 2 && (int)(gu_issued - gu_chunk) < NCH)
-                    gu_issue(ti, (int)(gu_issued - gu_chunk));
+                if (gu_issued == gu_chunk) gu_issue(ti, 0);  // not prefetched (a fused tile came before)
                 if (!wait_bar(tfull_bar(acc), acc_phase)) break;
                 fence_after();
                 bool stop = false;
 #pragma unroll 1
                 for (int c = 0; c < NCH; ++c) {
+                    // prefetch the next chunk (of this tile, or the first of the next tile)
+                    if (c + 1 < NCH) gu_issue(ti, c + 1);
+                    else if (t + tile_step < total_tiles) {
+                        const Tile tn = tile_at(t + tile_step);
+                        if (!(DW2 && tn.dw)) gu_issue(tn, 0);
+                    }
                     const int b = gu_chunk & 1;
                     if (!gu_wait(b, (gu_chunk >> 1) & 1)) { stop = true; break; }
-                    const uint8_t* gbuf = stg + (2 * b) * EPI_BUF_BYTES + lane * 64;
-                    const uint8_t* ubuf = gbuf + EPI_BUF_BYTES;
-                    float da[32];
+                    uint8_t* gbuf = stg + (2 * b) * EPI_BUF_BYTES + lane * 64;
+                    uint8_t* ubuf = gbuf + EPI_BUF_BYTES;
+                    float da[32], dG[32], dU[32];
                     tmem_ld32(tbase + 32 * c, da);
 #pragma unroll
                     for (int v = 0; v < 4; ++v) {
                         const int sw = (v ^ ((lane >> 1) & 3)) << 4;
-                        float G[8], U[8], dG[8], dU[8];
+                        float G[8], U[8];
                         unpack8(*reinterpret_cast<const uint4*>(gbuf + sw), G);
                         unpack8(*reinterpret_cast<const uint4*>(ubuf + sw), U);
 #pragma unroll
                         for (int i = 0; i < 8; ++i) {
                             const float sg = __fdividef(1.0f, 1.0f + __expf(-G[i]));
                             const float d = da[8 * v + i];
-                            dU[i] = d * G[i] * sg;
-                            dG[i] = d * U[i] * sg * (1.0f + G[i] * (1.0f - sg));
-                        }
-                        if (valid) {
-                            Vec<__nv_bfloat16>::store(dh + 32 * c + 8 * v, dG);
-                            Vec<__nv_bfloat16>::store(dh + F + 32 * c + 8 * v, dU);
+                            dU[8 * v + i] = d * G[i] * sg;
+                            dG[8 * v + i] = d * U[i] * sg * (1.0f + G[i] * (1.0f - sg));
                         }
                     }
-                    // every lane's reads of buffer b are done: order them before the async
-                    // proxy's next write into it, then load the chunk two ahead there
-                    fence_proxy_async();
+                    if (full_box) {
+                        store_row32_sw64(gbuf, lane, dG);
+                        store_row32_sw64(ubuf, lane, dU);
+                        fence_proxy_async();
+                        __syncwarp();
+                        if (lane == 0) {
+                            const uint32_t src = stg_u32 + (2 * b) * EPI_BUF_BYTES;
+                            tma_store_2d(&tmO0, src, ti.n0 + 32 * c, (int)grow0);
+                            tma_store_2d(&tmO0, src + EPI_BUF_BYTES, F + ti.n0 + 32 * c, (int)grow0);
+                            bulk_commit();
+                        }
+                    } else if (valid) {
+                        store_row32(dh + 32 * c, dG);
+                        store_row32(dh + F + 32 * c, dU);
+                    }
                     __syncwarp();
-                    Tile tn;
-                    int cn;
-                    if (ahead(c, 2, &tn, &cn)) gu_issue(tn, cn);
                     ++gu_chunk;
                 }
                 if (stop) break;
