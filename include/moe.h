@@ -170,6 +170,19 @@ moe_status moe_dispatch_noalloc(const moe_config* cfg, const int32_t* topk_idx, 
                                 void* x_perm, moe_stream_t stream);
 
 /*
+ * Row gather: dst[i] = src[rows[i]] for i < n_rows, rows of row_elems elements of dtype.
+ * The reordering between the blocks an expert host receives from the parties
+ * (source-major, Alg. 3 "send h to the host of idx") and the expert-major order its
+ * grouped GEMMs take, and back (Sec. 3.2: the gradient returned to each data owner).
+ *   src [n_src_rows, row_elems], dst [n_rows, row_elems]: device, 16-byte aligned,
+ *   row_elems * element size a multiple of 16 bytes; rows [n_rows] i32 device.
+ * A row index outside [0, n_src_rows) leaves that dst row untouched and is recorded as
+ * MOE_ERR_DEVICE_CHECK (moe_device_status). Bad sizes: MOE_ERR_INVALID_ARG.
+ */
+moe_status moe_gather_rows(const void* src, const int32_t* rows, int64_t n_rows, int64_t n_src_rows,
+                           int64_t row_elems, moe_dtype dtype, void* dst, moe_stream_t stream);
+
+/*
  * ForwardExpert of Alg. 6 for every routed expert, on its rows of x_perm, plus the
  * always-on shared experts on every token. Expert e is SwiGLU:
  *   [G|U] = x_perm_e W1[e]^T, A = silu(G) * U, Y = A W2[e]^T

@@ -80,6 +80,7 @@ _SIGS = {
     "moe_mse_loss": [_CFG] + [P] * 5 + [ctypes.c_size_t, P],
     "moe_expert_ffn_bwd_kernels": [_CFG, ctypes.POINTER(ctypes.c_int32)],
     "moe_sgd_update": [P, P, P, ctypes.c_int64, ctypes.c_int64, P, ctypes.c_float, ctypes.c_int, P],
+    "moe_gather_rows": [P, P, ctypes.c_int64, ctypes.c_int64, ctypes.c_int64, ctypes.c_int, P, P],
 }
 for _n, _a in _SIGS.items():
     f = getattr(_lib, _n)
@@ -217,6 +218,11 @@ def moe_mse_loss(cfg, out, target, loss, dout, workspace, workspace_bytes, strea
 def moe_sgd_update(w, dw, n_groups, group_elems, group_counts, lr, dtype, w_master=None, stream=None):
     _check(_lib.moe_sgd_update(_ptr(w), _ptr(dw), _ptr(w_master), int(n_groups), int(group_elems),
                                _ptr(group_counts), float(lr), int(dtype), _stream(stream)), "moe_sgd_update")
+
+
+def moe_gather_rows(src, rows, n_rows, n_src_rows, row_elems, dtype, dst, stream=None):
+    _check(_lib.moe_gather_rows(_ptr(src), _ptr(rows), int(n_rows), int(n_src_rows), int(row_elems),
+                                int(dtype), _ptr(dst), _stream(stream)), "moe_gather_rows")
 
 
 def moe_combine_fwd(cfg, y_perm, topk_w, slot_of, y_sh, out, stream=None):

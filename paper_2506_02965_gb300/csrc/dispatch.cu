@@ -204,6 +204,36 @@ __global__ void __launch_bounds__(256) gather_kernel(const T* __restrict__ x,
     }
 }
 
+// dst[i] = src[rows[i]] for n rows of `row_vecs` 16-byte vectors: one warp per row.
+// A row index outside [0, n_src) leaves dst[i] untouched and records
+// MOE_ERR_DEVICE_CHECK.
+__global__ void __launch_bounds__(256) gather_rows_kernel(const uint4* __restrict__ src,
+                                                          const int32_t* __restrict__ rows,
+                                                          int64_t n, int64_t n_src, int row_vecs,
+                                                          uint4* dst) {
+    pdl_begin();
+    const int lane = threadIdx.x & 31;
+    const int64_t i = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    if (i >= n) return;
+    const int64_t r = rows[i];
+    if (r < 0 || r >= n_src) {
+        if (lane == 0) record_status(MOE_ERR_DEVICE_CHECK);
+        return;
+    }
+    constexpr int U = 4;
+    const uint4* s = src + r * row_vecs;
+    uint4* o = dst + i * row_vecs;
+    for (int v0 = lane; v0 < row_vecs; v0 += 32 * U) {
+        uint4 buf[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u)
+            if (v0 + 32 * u < row_vecs) buf[u] = s[v0 + 32 * u];
+#pragma unroll
+        for (int u = 0; u < U; ++u)
+            if (v0 + 32 * u < row_vecs) o[v0 + 32 * u] = buf[u];
+    }
+}
+
 // out[t] = sum_j w[t,j] * y_perm[slot_of[t,j]] (+ sum_s y_sh[s,t]); fp32 accumulation.
 // One warp per token; every lane issues the loads of up to UB vectors of all k rows
 // before it uses any of them, so enough bytes are in flight to keep HBM busy.
@@ -557,6 +587,15 @@ cudaError_t launch_dispatch_noalloc(const int32_t* topk_idx, const void* x, int6
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     return launch_gather(x, slot_of, T, d, k, bf16, x_perm, s);
+}
+
+cudaError_t launch_gather_rows(const void* src, const int32_t* rows, int64_t n, int64_t n_src,
+                               int64_t row_bytes, void* dst, cudaStream_t s) {
+    if (n == 0) return cudaSuccess;
+    const unsigned blocks = (unsigned)((n + 7) / 8);
+    (void)launch_pdl(gather_rows_kernel, dim3(blocks), dim3(256), 0, s, (const uint4*)src, rows, n, n_src,
+                     (int)(row_bytes / 16), (uint4*)dst);
+    return cudaGetLastError();
 }
 
 cudaError_t dispatch_status(cudaStream_t s, int* code) { return tu_status_read_clear(s, code); }

@@ -682,6 +682,23 @@ moe_status moe_dispatch_bwd(const moe_config* cfg, const void* dx_perm, const in
                        "moe_dispatch_bwd");
 }
 
+moe_status moe_gather_rows(const void* src, const int32_t* rows, int64_t n_rows, int64_t n_src_rows,
+                           int64_t row_elems, moe_dtype dtype, void* dst, moe_stream_t stream) {
+    if (dtype != MOE_F32 && dtype != MOE_BF16) return fail(MOE_ERR_INVALID_ARG, "unknown dtype %d", (int)dtype);
+    if (n_rows < 0 || n_src_rows < 0 || row_elems < 0)
+        return fail(MOE_ERR_INVALID_ARG, "negative size (n_rows=%lld, n_src_rows=%lld, row_elems=%lld)",
+                    (long long)n_rows, (long long)n_src_rows, (long long)row_elems);
+    const int64_t row_bytes = row_elems * (dtype == MOE_BF16 ? 2 : 4);
+    if (row_bytes % 16) return fail(MOE_ERR_INVALID_ARG, "row of %lld bytes is not a multiple of 16", (long long)row_bytes);
+    if (n_rows == 0 || row_elems == 0) return MOE_OK;
+    REQUIRE_VEC(src);
+    REQUIRE(rows);
+    REQUIRE_VEC(dst);
+    if (row_bytes / 16 > INT32_MAX) return fail(MOE_ERR_INVALID_ARG, "row too long");
+    return cuda_status(launch_gather_rows(src, rows, n_rows, n_src_rows, row_bytes, dst, (cudaStream_t)stream),
+                       "moe_gather_rows");
+}
+
 moe_status moe_expert_ffn_bwd_kernels(const moe_config* cfg, int32_t* count) {
     moe_status st = check_cfg(cfg);
     if (st) return st;

@@ -69,6 +69,9 @@ cudaError_t launch_unpermute_reduce(const void* dx_perm, const int32_t* slot_of,
                                     const void* dx_router, const void* dx_sh, int S, int64_t T,
                                     int d, int k, bool bf16, void* dx, cudaStream_t s);
 cudaError_t dispatch_status(cudaStream_t s, int* code);
+// dst[i] = src[rows[i]] (row_bytes a multiple of 16)
+cudaError_t launch_gather_rows(const void* src, const int32_t* rows, int64_t n, int64_t n_src,
+                               int64_t row_bytes, void* dst, cudaStream_t s);
 // dispatch with its per-chunk counts in a fixed device array (no workspace argument)
 constexpr int64_t kNoAllocScratchInts = 1 << 16;  // 256 KiB of int32 chunk counts
 int64_t dispatch_noalloc_max_chunk_entries();

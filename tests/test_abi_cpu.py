@@ -111,6 +111,25 @@ def test_null_and_misaligned_pointers_rejected_on_host(L):
         L.moe_set_wait_limit_ns(0)
 
 
+def test_gather_rows_checks_arguments_on_host(L):
+    """moe_gather_rows rejects negative sizes, unknown dtypes, rows whose length is not a
+    multiple of 16 bytes (the kernel moves 16-byte vectors) and NULL or misaligned
+    pointers before any device work."""
+    cases = [((16, 16, -1, 4, 8, L.MOE_BF16, 16), "negative size"),
+             ((16, 16, 4, -1, 8, L.MOE_BF16, 16), "negative size"),
+             ((16, 16, 4, 4, 8, 9, 16), "dtype"),
+             ((16, 16, 4, 4, 6, L.MOE_BF16, 16), "multiple of 16"),
+             ((16, 16, 4, 4, 3, L.MOE_F32, 16), "multiple of 16"),
+             ((None, 16, 4, 4, 8, L.MOE_BF16, 16), "src is NULL"),
+             ((16, None, 4, 4, 8, L.MOE_BF16, 16), "rows is NULL"),
+             ((16, 16, 4, 4, 8, L.MOE_BF16, 24), "16-byte aligned")]
+    for args, frag in cases:
+        with pytest.raises(L.MoEError) as ei:
+            L.moe_gather_rows(*args, stream=0)
+        assert ei.value.status == L.MOE_ERR_INVALID_ARG and frag in L.moe_last_error(), frag
+    L.moe_gather_rows(None, None, 0, 0, 8, L.MOE_BF16, None, stream=0)  # nothing to move: OK
+
+
 def test_training_calls_check_arguments_on_host(L):
     """moe_sgd_update and moe_mse_loss reject bad arguments before any device work."""
     cases = [((16, 16, -1, 8, None, 0.1, L.MOE_BF16), "negative size"),
