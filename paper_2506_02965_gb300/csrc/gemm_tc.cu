@@ -311,12 +311,15 @@ __host__ __device__ constexpr uint32_t instr_desc() {
 }
 
 // Pipeline depth: as many operand stages as fit beside the epilogue's shared memory
-// (staging boxes, or the router's histogram), at most 12.
+// (staging boxes, or the router's histogram), at most 12. OCC CTAs share one SM (OCC = 2:
+// about half of the SM's 228 KiB each, for launches bound by their epilogue, whose
+// stores then come from twice as many warps per SM).
 __host__ __device__ constexpr int epi_extra_bytes(int epi) {
     return epi == 3 /* EPI_ROUTE */ ? 64 * 64 * 4 : 4 * EPI_STAGE_BYTES;
 }
-__host__ __device__ constexpr int num_stages(uint32_t stage_bytes, int epi) {
-    const int budget = 227 * 1024 - 1024 - 1024 - epi_extra_bytes(epi);  // dyn. smem, align, static
+__host__ __device__ constexpr int num_stages(uint32_t stage_bytes, int epi, int occ = 1) {
+    const int per_cta = occ == 1 ? 227 * 1024 : 112 * 1024;
+    const int budget = per_cta - 1024 - 1024 - epi_extra_bytes(epi);  // dyn. smem, align, static
     const int n = budget / (int)stage_bytes;
     return n > 12 ? 12 : n;
 }
@@ -521,8 +524,8 @@ __device__ __forceinline__ void route_epilogue_wide(const Params& p, const Tile&
 // for a weight gradient and the M-variable GEMM of the same backward step. (Interleaving
 // the two problems' tiles group by group measured slower: a tile with a long epilogue
 // followed by one with a short mainloop leaves the MMA waiting for an accumulator.)
-template <int BN, bool B_MN, bool VAR_K, int EPI, bool PAIR = false, bool DW2 = false>
-__global__ void __launch_bounds__(THREADS, 1)
+template <int BN, bool B_MN, bool VAR_K, int EPI, bool PAIR = false, bool DW2 = false, int OCC = 1>
+__global__ void __launch_bounds__(THREADS, OCC)
     grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA,
                         const __grid_constant__ CUtensorMap tmB,
                         const __grid_constant__ CUtensorMap tmO0,
@@ -532,6 +535,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                         const __grid_constant__ CUtensorMap tmO2, const Params p2) {
     pdl_begin();
     static_assert(!DW2 || (B_MN && !VAR_K && !PAIR && BN == 256), "fused: M-variable, MN-major B");
+    static_assert(OCC == 1 || (!PAIR && !DW2 && 2 * BN * OCC <= 512), "shared SMs: single-CTA tiles, TMEM for all");
     constexpr bool A_MN = VAR_K;
     constexpr int NPAIR = PAIR ? 2 : 1;
     constexpr int BNL = BN / NPAIR;  // B rows held by this CTA
@@ -541,7 +545,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     constexpr uint32_t A_BYTES = BM * KB * 2;
     constexpr uint32_t B_BYTES = BNL * KB * 2;
     constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
-    constexpr int NST = num_stages(STAGE_BYTES, EPI);
+    constexpr int NST = num_stages(STAGE_BYTES, EPI, OCC);
     constexpr uint32_t IDESC = instr_desc<BN, A_MN, B_MN, BMP>();
     constexpr uint32_t IDESC_DW = instr_desc<BN, true, true, BM>();
     constexpr int TMEM_COLS = (2 * BN <= 32) ? 32 : (2 * BN <= 64) ? 64 : (2 * BN <= 128) ? 128 : (2 * BN <= 256) ? 256 : 512;
@@ -1337,13 +1341,13 @@ static int band_for(int c) {
     return b;
 }
 
-template <int BN, bool B_MN, bool VAR_K, int EPI, bool PAIR = false, bool DW2 = false>
+template <int BN, bool B_MN, bool VAR_K, int EPI, bool PAIR = false, bool DW2 = false, int OCC = 1>
 static cudaError_t launch(const CUtensorMap& ma, const CUtensorMap& mb, const CUtensorMap& mo0,
                           const CUtensorMap& mo1, const Params& p, int64_t tiles_ub,
                           cudaStream_t s, const CUtensorMap* ma2 = nullptr,
                           const CUtensorMap* mb2 = nullptr, const CUtensorMap* mo2 = nullptr,
                           const Params* p2 = nullptr) {
-    auto kern = grouped_gemm_kernel<BN, B_MN, VAR_K, EPI, PAIR, DW2>;
+    auto kern = grouped_gemm_kernel<BN, B_MN, VAR_K, EPI, PAIR, DW2, OCC>;
     const CUtensorMap& A2 = ma2 ? *ma2 : ma;
     const CUtensorMap& B2 = mb2 ? *mb2 : mb;
     const CUtensorMap& O2 = mo2 ? *mo2 : mo0;
@@ -1352,7 +1356,7 @@ static cudaError_t launch(const CUtensorMap& ma, const CUtensorMap& mb, const CU
     constexpr int NPAIR = PAIR ? 2 : 1;
     constexpr int KB = kblock_rows(VAR_K, PAIR);
     constexpr int STB = BM * KB * 2 + BN / NPAIR * KB * 2;  // bytes of one operand stage
-    constexpr int NST = num_stages((uint32_t)STB, EPI);
+    constexpr int NST = num_stages((uint32_t)STB, EPI, OCC);
     const int extra_max = EPI == EPI_ROUTE ? 64 * 64 * 4 : EPI_WARPS * epi_stage_bytes(EPI);
     const int extra = EPI == EPI_ROUTE ? p.hist_n * 4 : EPI_WARPS * epi_stage_bytes(EPI);
     const int smem_max = NST * STB + 1024 + extra_max;
@@ -1405,7 +1409,7 @@ static cudaError_t launch(const CUtensorMap& ma, const CUtensorMap& mb, const CU
         cfg.numAttrs = 2;
         return cudaLaunchKernelEx(&cfg, kern, ma, mb, mo0, mo1, P1, A2, B2, O2, P2);
     } else {
-        const int grid = (int)std::min<int64_t>(tiles_ub, sm_count());
+        const int grid = (int)std::min<int64_t>(tiles_ub, (int64_t)OCC * sm_count());
         P1.band = P2.band = band_for(grid);
         (void)launch_pdl(kern, dim3(grid), dim3(THREADS), smem, s, ma, mb, mo0, mo1, P1, A2, B2, O2, P2);
         return cudaGetLastError();
@@ -1523,6 +1527,8 @@ cudaError_t launch_gemm_m(const GemmMArgs& g, bool bf16, cudaStream_t s) {
         return launch<128, true, false, EPI_SWIGLU_BWD>(ma, mb, mo0, mo1, p, mt_ub * (g.N / 128), s);
     }
     if (!make_map(&mo0, g.out0, g.N, o_rows, 0, true)) return cudaErrorInvalidValue;
+    if (g.slim && g.N % 128 == 0)
+        return launch<128, true, false, EPI_STORE, false, false, 2>(ma, mb, mo0, mo0, p, mt_ub * (g.N / 128), s);
     if (g.N % 256 == 0) {
         if (pair) return launch<256, true, false, EPI_STORE, true>(ma, mb, mo0, mo0, p, pt_ub * (g.N / 256), s);
         return launch<256, true, false, EPI_STORE>(ma, mb, mo0, mo0, p, mt_ub * (g.N / 256), s);

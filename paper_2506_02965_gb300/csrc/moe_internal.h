@@ -118,6 +118,9 @@ struct GemmMArgs {
     void* out0;
     void* out1;
     const void* aux;
+    // EPI_STORE with MN-major B and N % 128 == 0: two CTAs per SM with 128-wide tiles, for
+    // a short contraction whose time is the epilogue's stores (the router's dx_router)
+    bool slim;
 };
 
 // C_g[M, N] = sum over the rows r of group g of A[r, m] * B[r, n]  (K varies per group)

@@ -769,6 +769,7 @@ static cudaError_t launch_route_bwd_tc(const RouteBwdArgs& a, void* ws, cudaStre
         m.b_rows = a.E;
         m.epi = EPI_STORE;
         m.out0 = a.dx_router;
+        m.slim = true;  // one k-block per tile: the stores bound it
         return launch_gemm_m(m, true, s);
     }
     return cudaSuccess;
