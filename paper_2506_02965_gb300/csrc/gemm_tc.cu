@@ -37,7 +37,8 @@ constexpr int EPI_BUF_BYTES = EPI_BOX * EPI_BOX * 2;
 // backward 2 x (G, U) boxes
 constexpr int EPI_NBUF = 4;
 constexpr int EPI_STAGE_BYTES = EPI_NBUF * EPI_BUF_BYTES;
-__host__ __device__ constexpr int epi_stage_bytes(int) { return EPI_STAGE_BYTES; }
+// per epilogue warp (the router-gradient partials are stored straight from registers)
+__host__ __device__ constexpr int epi_stage_bytes(int epi) { return epi == EPI_DWR ? 0 : EPI_STAGE_BYTES; }
 constexpr int MAX_GROUPS = 256;
 
 struct Params {
@@ -315,7 +316,7 @@ __host__ __device__ constexpr uint32_t instr_desc() {
 // about half of the SM's 228 KiB each, for launches bound by their epilogue, whose
 // stores then come from twice as many warps per SM).
 __host__ __device__ constexpr int epi_extra_bytes(int epi) {
-    return epi == 3 /* EPI_ROUTE */ ? 64 * 64 * 4 : 4 * EPI_STAGE_BYTES;
+    return epi == EPI_ROUTE ? 64 * 64 * 4 : EPI_WARPS * epi_stage_bytes(epi);
 }
 __host__ __device__ constexpr int num_stages(uint32_t stage_bytes, int epi, int occ = 1) {
     const int per_cta = occ == 1 ? 227 * 1024 : 112 * 1024;
@@ -1567,8 +1568,10 @@ cudaError_t launch_gemm_k(const GemmKArgs& g, bool bf16, cudaStream_t s) {
     if (g.epi == EPI_DWR) {  // fp32 partials, N = 64, 128 or 256 (experts, zero-padded)
         if ((g.N != 64 && g.N != 128 && g.N != 256) || g.M % BM) return cudaErrorInvalidValue;
         p.E = g.E;
-        if (g.N == 64) return launch<64, true, true, EPI_DWR>(ma, mb, ma, ma, p, tiles, s);
-        if (g.N == 128) return launch<128, true, true, EPI_DWR>(ma, mb, ma, ma, p, tiles, s);
+        // two CTAs per SM where TMEM allows: each streams its token chunk of x from HBM at
+        // a per-CTA rate, and every tile is resident in one round
+        if (g.N == 64) return launch<64, true, true, EPI_DWR, false, false, 2>(ma, mb, ma, ma, p, tiles, s);
+        if (g.N == 128) return launch<128, true, true, EPI_DWR, false, false, 2>(ma, mb, ma, ma, p, tiles, s);
         return launch<256, true, true, EPI_DWR>(ma, mb, ma, ma, p, tiles, s);
     }
     if (!make_map(&mo, g.out, g.N, (int64_t)g.G * g.M, 0, true)) return cudaErrorInvalidValue;
