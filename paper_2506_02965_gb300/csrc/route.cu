@@ -635,8 +635,8 @@ struct RbTcLayout {
     size_t dw, db, off, dz, total;
 };
 // Tokens per chunk of the chunked dW_r contraction: about 256 tiles of 128 model columns
-// in all (one wave of 152 measured slower), at most 128 - P chunks (the grouped GEMM's
-// group limit), a multiple of 64.
+// in all (one wave of 152 single-CTA tiles measured slower), at most 128 - P chunks
+// (well inside the grouped GEMM's 256 groups), a multiple of 64.
 static RbTcLayout rb_tc_layout(int64_t T, int P, int E, int d) {
     RbTcLayout L;
     const int64_t mt = std::max(1, d / 128);
