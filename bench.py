@@ -13,8 +13,9 @@ step).
   python bench.py --impl reference ...   # the fp64 CPU oracle on the host cores
 
 Timing: W untimed warm-up steps, then K steps timed one by one with CUDA events on
-the launching stream; L2 is flushed (a 256 MiB write, outside the events) before
-every timed step. Under torchrun each rank runs its own replica (the layer does not
+the launching stream; L2 is flushed (a 256 MiB write, then a 256 MiB read of another
+buffer so that no dirty line is written back inside the step; both outside the events)
+before every timed step. Under torchrun each rank runs its own replica (the layer does not
 shard; no collective on the data path); the time is the max over ranks and the
 value is the tokens of all ranks per second. Prints one JSON line on rank 0.
 
@@ -422,10 +423,15 @@ def main():
     for name in ("w1", "w2", "ws1", "ws2"):  # on the device now; x and dOut stay for e2e
         inp.pop(name, None)
     flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+    # after the flush write, a read of another buffer larger than L2 leaves it holding
+    # clean lines: the timed call then starts cold without paying for the write-back of
+    # the flush's dirty lines
+    clean = torch.ones(FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
     stream = torch.cuda.current_stream()
 
     for i in range(max(3, a.warmup)):
         flush.fill_(i & 0xFF)
+        clean.sum()
         lay.step()
     torch.cuda.synchronize()
     lay.check_status()
@@ -441,6 +447,7 @@ def main():
     t_wall = time.perf_counter()
     for i in range(K):
         flush.fill_(i & 0xFF)
+        clean.sum()
         ev[i][0].record(stream)
         lay.step()
         ev[i][1].record(stream)
@@ -458,10 +465,6 @@ def main():
     names = [n for n, _ in lay.STAGES]
     evs = [{n: (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
             for n in names} for _ in range(Ks)]
-    # after the flush write, a read of another buffer larger than L2 leaves it holding
-    # clean lines: the timed call then starts cold without paying for the write-back of
-    # the flush's dirty lines
-    clean = torch.ones(FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
     barrier()
     torch.cuda.synchronize()
     for i in range(Ks):
@@ -554,7 +557,8 @@ def main():
         "data": "synthetic (seeded numpy PCG64, workload shapes, random-init weights)",
         "config": {"workload": workload_desc(sh), "global_batch": world * sh.T,
                    "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
-                   "l2": "flushed (256 MiB write) before every timed step"},
+                   "l2": "flushed before every timed step (256 MiB write, then a 256 MiB read so "
+                         "that no dirty line is left)"},
         "roofline": roofline,
         "roofline_mem": {"bound": "hbm", "achieved": mem_bytes / (mem_ms / 1e3) / 1e9,
                          "peak": pk["hbm_gbs"], "unit": "GB/s",
