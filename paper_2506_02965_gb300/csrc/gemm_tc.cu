@@ -345,6 +345,9 @@ struct Tile {
 // logits of its token, adds the party's bias, writes logits and Softmax
 // probabilities, picks the k largest logits (equal logits: lower expert id first),
 // writes the gate weights p[I] (renormalised on request) and counts the picks.
+// The loops over experts are unrolled (the logits live in registers); the loop over
+// the k picks is not: each tile runs this code once per CTA, so it runs from a cold
+// instruction cache, and an unrolled 8 x BN selection was fetch-bound (k = 6, E = 64).
 template <int BN>
 __device__ __forceinline__ void route_epilogue(const Params& p, const Tile& ti, int m, bool valid,
                                                uint32_t tbase, int* hist) {
@@ -367,10 +370,13 @@ __device__ __forceinline__ void route_epilogue(const Params& p, const Tile& ti, 
             mx = fmaxf(mx, z[e]);
         }
     }
+    float ez[BN];
     float sum = 0.f;
 #pragma unroll
-    for (int e = 0; e < BN; ++e)
-        if (e < E) sum += expf(z[e] - mx);
+    for (int e = 0; e < BN; ++e) {
+        ez[e] = e < E ? expf(z[e] - mx) : 0.f;
+        if (e < E) sum += ez[e];
+    }
     float* lg = (float*)p.out0 + t * E;
     float* pr = (float*)p.out1 + t * E;
 #pragma unroll
@@ -378,41 +384,34 @@ __device__ __forceinline__ void route_epilogue(const Params& p, const Tile& ti, 
         if (e < E) {
             *reinterpret_cast<float4*>(lg + e) = make_float4(z[e], z[e + 1], z[e + 2], z[e + 3]);
             *reinterpret_cast<float4*>(pr + e) =
-                make_float4(expf(z[e] - mx) / sum, expf(z[e + 1] - mx) / sum,
-                            expf(z[e + 2] - mx) / sum, expf(z[e + 3] - mx) / sum);
+                make_float4(ez[e] / sum, ez[e + 1] / sum, ez[e + 2] / sum, ez[e + 3] / sum);
         }
     }
     uint64_t taken = 0;
     float wsum = 0.f;
-    int sel[8];
-    float wsel[8];
+    int32_t* ti_out = p.topk_idx + t * k;
+    float* tw_out = p.topk_w + t * k;
+#pragma unroll 1
+    for (int j = 0; j < k; ++j) {
+        int bi = -1;
+        float bv = 0.f;
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
-        sel[j] = 0;
-        wsel[j] = 0.f;
-        if (j < k) {
-            int bi = -1;
-            float bv = 0.f;
-#pragma unroll
-            for (int e = 0; e < BN; ++e) {
-                if (e < E && !((taken >> e) & 1ull) && (bi < 0 || z[e] > bv)) {
-                    bi = e;
-                    bv = z[e];
-                }
+        for (int e = 0; e < BN; ++e) {
+            if (e < E && !((taken >> e) & 1ull) && (bi < 0 || z[e] > bv)) {
+                bi = e;
+                bv = z[e];
             }
-            taken |= 1ull << bi;
-            sel[j] = bi;
-            wsel[j] = expf(bv - mx) / sum;
-            wsum += wsel[j];
         }
+        taken |= 1ull << bi;
+        const float w = expf(bv - mx) / sum;
+        wsum += w;
+        ti_out[j] = bi;
+        tw_out[j] = w;
+        atomicAdd(&hist[ti.g * E + bi], 1);
     }
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-        if (j < k) {
-            p.topk_idx[t * k + j] = sel[j];
-            p.topk_w[t * k + j] = p.normalize ? wsel[j] / wsum : wsel[j];
-            atomicAdd(&hist[ti.g * E + sel[j]], 1);
-        }
+    if (p.normalize) {
+#pragma unroll 1
+        for (int j = 0; j < k; ++j) tw_out[j] = tw_out[j] / wsum;
     }
 }
 
