@@ -566,7 +566,10 @@ __global__ void __launch_bounds__(THREADS, OCC)
     const int tile0 = (int)blockIdx.x / NPAIR, tile_step = (int)gridDim.x / NPAIR;
 
     // group -> tile prefix
-    const int tiles_n = (EPI == EPI_SWIGLU_FWD) ? p.N / 256 : (EPI == EPI_ROUTE) ? 1 : p.N / BN;
+    // N-tiles per row of tiles; the last one may be ragged (N a multiple of 128 with
+    // 256-wide tiles: its columns past N are computed from zero-filled or unused operand
+    // columns and never stored)
+    const int tiles_n = (EPI == EPI_SWIGLU_FWD) ? p.N / 256 : (EPI == EPI_ROUTE) ? 1 : (p.N + BN - 1) / BN;
     if (threadIdx.x == 0) {
         int acc = 0;
         for (int g = 0; g < p.G; ++g) {
@@ -1119,14 +1122,15 @@ __global__ void __launch_bounds__(THREADS, OCC)
                 const int F = p.F;
                 __nv_bfloat16* dh = (__nv_bfloat16*)p.out0 + (ti.out_row + m) * (int64_t)(2 * F) + ti.n0;
                 constexpr int NCH = BN / 32;
+                const int nchv = min(NCH, (F - ti.n0) / 32);  // chunks inside F (a ragged last tile)
                 if (gu_issued == gu_chunk) gu_issue(ti, 0);  // not prefetched (a fused tile came before)
                 if (!wait_bar(tfull_bar(acc), acc_phase)) break;
                 fence_after();
                 bool stop = false;
 #pragma unroll 1
-                for (int c = 0; c < NCH; ++c) {
+                for (int c = 0; c < nchv; ++c) {
                     // prefetch the next chunk (of this tile, or the first of the next tile)
-                    if (c + 1 < NCH) gu_issue(ti, c + 1);
+                    if (c + 1 < nchv) gu_issue(ti, c + 1);
                     else if (t + tile_step < total_tiles) {
                         const Tile tn = tile_at(t + tile_step);
                         if (!(DW2 && tn.dw)) gu_issue(tn, 0);
@@ -1225,7 +1229,7 @@ __global__ void __launch_bounds__(THREADS, OCC)
                     else
                         out = (__nv_bfloat16*)p.out0 + (ti.out_row + m) * (int64_t)p.N;
 #pragma unroll 1
-                    for (int c = 0; c < BN; c += 32) {
+                    for (int c = 0; c < BN && ti.n0 + c < p.N; c += 32) {
                         float y[32];
                         if (ti.k_iters > 0) {
                             tmem_ld32(tbase + c, y);
@@ -1433,14 +1437,14 @@ void set_gemm_pairs(int mode) { tc::g_pairs = mode; }
 // and pairs win (d = 4096: the expert backward 17.8 -> 17.2 ms; d = 1024: +4%).
 bool gemm_m_uses_pairs(const GemmMArgs& g) {
     using namespace tc;
-    if (g.N % 256 != 0) return false;
+    if (g.N % 128 != 0) return false;  // 256-wide pair tiles, the last one possibly ragged
     if (g_pairs == MOE_PAIRS_ALL) return true;
     if (g_pairs != MOE_PAIRS_AUTO) return false;
     if (g.epi == EPI_SWIGLU_BWD && g.K < 2048) return false;
     if (g.epi == EPI_STORE && !g.b_kmajor && g.K >= 512) return true;
     const int64_t pt_ub = g.rows.offsets ? ((int64_t)g.rows.rows + 2 * BM - 1) / (2 * BM) + g.G
                                          : (int64_t)g.G * ((g.rows.rows + 2 * BM - 1) / (2 * BM));
-    return pt_ub * (g.N / 256) >= 4 * (int64_t)(sm_count() / 2);
+    return pt_ub * ((g.N + 255) / 256) >= 4 * (int64_t)(sm_count() / 2);
 }
 
 // K-variable weight gradients (dW = A^T B over each group's rows) as 256 x 256 CTA-pair
@@ -1448,10 +1452,10 @@ bool gemm_m_uses_pairs(const GemmMArgs& g) {
 // pair tiles.
 bool gemm_k_uses_pairs(const GemmKArgs& g) {
     using namespace tc;
-    if (g.epi != EPI_STORE || g.M % 256 != 0 || g.N % 256 != 0) return false;
+    if (g.epi != EPI_STORE || g.M % 256 != 0 || g.N % 128 != 0) return false;
     if (g_pairs == MOE_PAIRS_ALL) return true;
     if (g_pairs != MOE_PAIRS_AUTO) return false;
-    return (int64_t)g.G * (g.M / 256) * (g.N / 256) >= 4 * (int64_t)(sm_count() / 2);
+    return (int64_t)g.G * (g.M / 256) * ((g.N + 255) / 256) >= 4 * (int64_t)(sm_count() / 2);
 }
 
 // M-variable grouped GEMM (forward, dA, dX).
@@ -1502,11 +1506,11 @@ cudaError_t launch_gemm_m(const GemmMArgs& g, bool bf16, cudaStream_t s) {
     if (g.epi == EPI_STORE && g.b_kmajor) {  // Y = A W2^T: B = W2[e] as [N=d, K=F]
         p.b_group_rows = g.N;
         if (!make_map(&mo0, g.out0, g.N, o_rows, 0, true)) return cudaErrorInvalidValue;
+        if (pair) {
+            if (!make_map(&mb, g.b, g.K, (int64_t)g.G * g.N, 128)) return cudaErrorInvalidValue;
+            return launch<256, false, false, EPI_STORE, true>(ma, mb, mo0, mo0, p, pt_ub * ((g.N + 255) / 256), s);
+        }
         if (g.N % 256 == 0) {
-            if (pair) {
-                if (!make_map(&mb, g.b, g.K, (int64_t)g.G * g.N, 128)) return cudaErrorInvalidValue;
-                return launch<256, false, false, EPI_STORE, true>(ma, mb, mo0, mo0, p, pt_ub * (g.N / 256), s);
-            }
             if (!make_map(&mb, g.b, g.K, (int64_t)g.G * g.N, 256)) return cudaErrorInvalidValue;
             return launch<256, false, false, EPI_STORE>(ma, mb, mo0, mo0, p, mt_ub * (g.N / 256), s);
         }
@@ -1520,19 +1524,16 @@ cudaError_t launch_gemm_m(const GemmMArgs& g, bool bf16, cudaStream_t s) {
         p.F = g.N;
         if (!make_map(&mo0, g.out0, 2 * (int64_t)g.N, o_rows, 0, true)) return cudaErrorInvalidValue;
         if (!make_map(&mo1, g.aux, 2 * (int64_t)g.N, o_rows, 0, true)) return cudaErrorInvalidValue;
-        if (g.N % 256 == 0) {
-            if (pair) return launch<256, true, false, EPI_SWIGLU_BWD, true>(ma, mb, mo0, mo1, p, pt_ub * (g.N / 256), s);
-            return launch<256, true, false, EPI_SWIGLU_BWD>(ma, mb, mo0, mo1, p, mt_ub * (g.N / 256), s);
-        }
+        if (pair)
+            return launch<256, true, false, EPI_SWIGLU_BWD, true>(ma, mb, mo0, mo1, p, pt_ub * ((g.N + 255) / 256), s);
+        if (g.N % 256 == 0) return launch<256, true, false, EPI_SWIGLU_BWD>(ma, mb, mo0, mo1, p, mt_ub * (g.N / 256), s);
         return launch<128, true, false, EPI_SWIGLU_BWD>(ma, mb, mo0, mo1, p, mt_ub * (g.N / 128), s);
     }
     if (!make_map(&mo0, g.out0, g.N, o_rows, 0, true)) return cudaErrorInvalidValue;
     if (g.slim && g.N % 128 == 0)
         return launch<128, true, false, EPI_STORE, false, false, 2>(ma, mb, mo0, mo0, p, mt_ub * (g.N / 128), s);
-    if (g.N % 256 == 0) {
-        if (pair) return launch<256, true, false, EPI_STORE, true>(ma, mb, mo0, mo0, p, pt_ub * (g.N / 256), s);
-        return launch<256, true, false, EPI_STORE>(ma, mb, mo0, mo0, p, mt_ub * (g.N / 256), s);
-    }
+    if (pair) return launch<256, true, false, EPI_STORE, true>(ma, mb, mo0, mo0, p, pt_ub * ((g.N + 255) / 256), s);
+    if (g.N % 256 == 0) return launch<256, true, false, EPI_STORE>(ma, mb, mo0, mo0, p, mt_ub * (g.N / 256), s);
     return launch<128, true, false, EPI_STORE>(ma, mb, mo0, mo0, p, mt_ub * (g.N / 128), s);
 }
 
@@ -1575,7 +1576,7 @@ cudaError_t launch_gemm_k(const GemmKArgs& g, bool bf16, cudaStream_t s) {
     }
     if (!make_map(&mo, g.out, g.N, (int64_t)g.G * g.M, 0, true)) return cudaErrorInvalidValue;
     if (pair)
-        return launch<256, true, true, EPI_STORE, true>(ma, mb, mo, mo, p, (int64_t)g.G * (g.M / 256) * (g.N / 256), s);
+        return launch<256, true, true, EPI_STORE, true>(ma, mb, mo, mo, p, (int64_t)g.G * (g.M / 256) * ((g.N + 255) / 256), s);
     if (g.N % 256 == 0) return launch<256, true, true, EPI_STORE>(ma, mb, mo, mo, p, tiles * (g.N / 256), s);
     return launch<128, true, true, EPI_STORE>(ma, mb, mo, mo, p, tiles * (g.N / 128), s);
 }

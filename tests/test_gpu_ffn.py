@@ -145,12 +145,15 @@ def test_expert_ffn_is_deterministic(L):
 def test_expert_ffn_single_cta_and_pair_tiles(L, pairs):
     """The 256-wide GEMMs in every tile mode: one CTA per 128x256 tile, a CTA pair per
     256x256 tile, or the automatic choice per launch (ragged experts, an empty expert, a
-    skewed split, experts ending at every offset of a k-block)."""
+    skewed split, experts ending at every offset of a k-block; d and F of 128 mod 256, so
+    that the last pair tile of dA, dW2, GEMM2, dX and dW1 along N holds 128 columns)."""
     L.moe_set_gemm_pairs(pairs)
     try:
         for case in [(777, 512, 8, 512, 2, "skewed", "bf16", 0, 0),
                      (300, 256, 4, 256, 2, "uniform", "bf16", 1, 256),
                      (1024, 1024, 16, 2816, 2, "uniform", "bf16", 0, 0),
+                     (777, 384, 8, 384, 2, "skewed", "bf16", 1, 640),
+                     (512, 1024, 4, 1408, 2, "skewed", "bf16", 0, 0),
                      # experts of 0, 1, 15, 16, 17, 63, 64, 65, 127, 128, 129, 200, 255, 256,
                      # 257 rows: every way the weight gradients' last k-block (64 rows, 128 for
                      # pair tiles) can end (pairs: zeroed on both CTAs)
