@@ -27,6 +27,10 @@ constexpr int BK = 64;  // 64 bf16 = 128 bytes = one 128B-swizzle row
 // gradients), whose operands are both MN-major (64-element TMA boxes): 128-row boxes
 // there halve the boxes and stage hand-offs per byte (3 stages of 64 KiB per CTA).
 __host__ __device__ constexpr int kblock_rows(bool var_k, bool pair) { return (var_k && pair) ? 128 : BK; }
+// k-blocks per operand stage: 2 for the router up to 64 experts (its stream of x is bound
+// by a fixed cost per stage hand-off, so a stage carries two 64-wide boxes of each
+// operand; wider B would leave too few stages), else 1
+__host__ __device__ constexpr int kblocks_per_stage(int epi, int bn) { return (epi == 3 /* EPI_ROUTE */ && bn <= 64) ? 2 : 1; }
 constexpr int STAGES = 4;
 constexpr int EPI_WARPS = 4;
 constexpr int THREADS = 64 + 32 * EPI_WARPS;  // TMA warp, MMA warp, epilogue warps
@@ -66,6 +70,9 @@ struct Params {
     int32_t* topk_idx;
     float* topk_w;
     int32_t* counts;
+    // EPI_ROUTE: token rows per tile (1..BM; the A box height), so that the tiles of a
+    // short batch spread over every SM (each CTA streams its rows at a per-CTA rate)
+    int tile_rows;
 };
 
 // ------------------------------------------------------------------------ PTX helpers
@@ -542,8 +549,11 @@ __global__ void __launch_bounds__(THREADS, OCC)
     constexpr int BMP = BM * NPAIR;  // rows of one (pair) tile
     constexpr int KB = kblock_rows(VAR_K, PAIR);  // contraction rows per k-block
     constexpr uint32_t ATOM = KB * 128;              // bytes of one 64-wide MN-major box
-    constexpr uint32_t A_BYTES = BM * KB * 2;
-    constexpr uint32_t B_BYTES = BNL * KB * 2;
+    constexpr int KPS = kblocks_per_stage(EPI, BN);
+    constexpr uint32_t A_BOX = BM * KB * 2;   // one k-block of A
+    constexpr uint32_t B_BOX = BNL * KB * 2;  // one k-block of B
+    constexpr uint32_t A_BYTES = A_BOX * KPS;
+    constexpr uint32_t B_BYTES = B_BOX * KPS;
     constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
     constexpr int NST = num_stages(STAGE_BYTES, EPI, OCC);
     constexpr uint32_t IDESC = instr_desc<BN, A_MN, B_MN, BMP>();
@@ -579,7 +589,8 @@ __global__ void __launch_bounds__(THREADS, OCC)
                 mt = p.Mout / BMP;
             } else {
                 const int rows = p.offsets ? (p.offsets[g + 1] - p.offsets[g]) : p.rows;
-                mt = rows > 0 ? (rows + BMP - 1) / BMP : 0;
+                const int rpt = (EPI == EPI_ROUTE) ? p.tile_rows : BMP;  // rows per tile
+                mt = rows > 0 ? (rows + rpt - 1) / rpt : 0;
             }
             acc += mt * tiles_n;
         }
@@ -676,7 +687,7 @@ __global__ void __launch_bounds__(THREADS, OCC)
         band_split(local, mt_g, tiles_n, group_band(p, rows_g, mt_g), &mt, &nt);
         ti.g = g;
         ti.we = p.gexp ? p.gexp[g] : g;
-        ti.m0 = mt * BMP + (int)rank * BM;
+        ti.m0 = (EPI == EPI_ROUTE) ? mt * p.tile_rows : mt * BMP + (int)rank * BM;
         ti.n0 = nt * ((EPI == EPI_SWIGLU_FWD) ? 128 : BN);
         int64_t r0, nrows, a0, b0, o0;
         if (p.offsets) {
@@ -697,11 +708,12 @@ __global__ void __launch_bounds__(THREADS, OCC)
             ti.k_iters = (int)((nrows + KB - 1) / KB);
             ti.last_rows = (int)(nrows - (int64_t)(ti.k_iters - 1) * KB);
         } else {
-            ti.mvalid = (int)nrows;
+            // router tiles of tile_rows rows: the box's rows past them are the next tile's
+            ti.mvalid = (EPI == EPI_ROUTE) ? (int)min64(nrows, (int64_t)ti.m0 + p.tile_rows) : (int)nrows;
             ti.a_row = a0;
             ti.b_row = 0;
             ti.out_row = o0;
-            ti.k_iters = p.K / BK;
+            ti.k_iters = p.K / (BK * KPS);
             ti.last_rows = BK;
         }
         return ti;
@@ -826,13 +838,16 @@ __global__ void __launch_bounds__(THREADS, OCC)
                             parmed |= 1u << stage;
                             pnext ^= 1u << stage;
                         }
+                    } else if constexpr (EPI == EPI_ROUTE) {
+                        mbar_expect_tx(fb, (uint32_t)p.tile_rows * 128u * KPS + B_BYTES);  // A boxes of tile_rows rows
                     } else {
                         mbar_expect_tx(fb, STAGE_BYTES);
                     }
-                    const int k0 = kb * KB;
+                    const int k0 = kb * KB * KPS;
                     const bool dw = DW2 && ti.dw;
                     if (!A_MN && !dw) {
-                        load(sa, &tmA, fb, k0, (int)(ti.a_row + ti.m0));
+#pragma unroll
+                        for (int i = 0; i < KPS; ++i) load(sa + i * A_BOX, &tmA, fb, k0 + KB * i, (int)(ti.a_row + ti.m0));
                     } else {
                         const CUtensorMap* mA = dw ? &tmA2 : &tmA;
 #pragma unroll
@@ -850,7 +865,10 @@ __global__ void __launch_bounds__(THREADS, OCC)
                             load(sb + 128 * 128, &tmB, fb, k0, (int)(r + p.F));
                         }
                     } else if (!B_MN) {
-                        load(sb, &tmB, fb, k0, (int)((int64_t)ti.we * p.b_group_rows + ti.n0 + rank * BNL));
+#pragma unroll
+                        for (int i = 0; i < KPS; ++i)
+                            load(sb + i * B_BOX, &tmB, fb, k0 + KB * i,
+                                 (int)((int64_t)ti.we * p.b_group_rows + ti.n0 + rank * BNL));
                     } else {
                         const int64_t krow = (VAR_K || dw) ? (ti.b_row + k0) : ((int64_t)ti.we * p.b_group_rows + k0);
                         const CUtensorMap* mB = dw ? &tmB2 : &tmB;
@@ -918,7 +936,7 @@ __global__ void __launch_bounds__(THREADS, OCC)
                 // group. Only K=16 steps that contain valid rows are issued, and inside the
                 // last of them the A rows past the group's end are zeroed (A alone suffices:
                 // their products with any finite B row vanish).
-                int ksteps = KB / 16;
+                int ksteps = KB * KPS / 16;
                 const bool dwt = DW2 && ti.dw;
                 if ((VAR_K || dwt) && kb == ti.k_iters - 1 && ti.last_rows < KB) {
                     ksteps = (ti.last_rows + 15) / 16;
@@ -938,12 +956,12 @@ __global__ void __launch_bounds__(THREADS, OCC)
                 fence_after();
                 if (lane == 0) {
 #pragma unroll
-                    for (int kk = 0; kk < KB / 16; ++kk) {
+                    for (int kk = 0; kk < KB * KPS / 16; ++kk) {
                         if (kk >= ksteps) break;
                         uint64_t ad, bd;
-                        if (!A_MN && !dwt) ad = smem_desc(sa + kk * 32, 16, 1024);
+                        if (!A_MN && !dwt) ad = smem_desc(sa + (kk / (KB / 16)) * A_BOX + (kk % (KB / 16)) * 32, 16, 1024);
                         else ad = smem_desc(sa + kk * 2048, ATOM, 1024);
-                        if (!B_MN) bd = smem_desc(sb + kk * 32, 16, 1024);
+                        if (!B_MN) bd = smem_desc(sb + (kk / (KB / 16)) * B_BOX + (kk % (KB / 16)) * 32, 16, 1024);
                         else bd = smem_desc(sb + kk * 2048, ATOM, 1024);
                         if constexpr (PAIR) mma_bf16_pair(tmem_d, ad, bd, IDESC, (kb | kk) ? 1u : 0u);
                         else mma_bf16(tmem_d, ad, bd, dwt ? IDESC_DW : IDESC, (kb | kk) ? 1u : 0u);
@@ -1359,7 +1377,7 @@ static cudaError_t launch(const CUtensorMap& ma, const CUtensorMap& mb, const CU
     Params P2 = p2 ? *p2 : p;
     constexpr int NPAIR = PAIR ? 2 : 1;
     constexpr int KB = kblock_rows(VAR_K, PAIR);
-    constexpr int STB = BM * KB * 2 + BN / NPAIR * KB * 2;  // bytes of one operand stage
+    constexpr int STB = (BM * KB * 2 + BN / NPAIR * KB * 2) * kblocks_per_stage(EPI, BN);  // bytes of one operand stage
     constexpr int NST = num_stages((uint32_t)STB, EPI, OCC);
     const int extra_max = EPI == EPI_ROUTE ? 64 * 64 * 4 : EPI_WARPS * epi_stage_bytes(EPI);
     const int extra = EPI == EPI_ROUTE ? p.hist_n * 4 : EPI_WARPS * epi_stage_bytes(EPI);
@@ -1673,10 +1691,14 @@ cudaError_t launch_route_tc(const RouteArgs& a, cudaStream_t s) {
     const int BNr = a.E <= 16 ? 16 : a.E <= 32 ? 32 : a.E <= 64 ? 64 : a.E <= 128 ? 128 : 256;
     if (a.E > 256) return cudaErrorInvalidValue;
     p.N = BNr;
+    // rows per tile: the batch split evenly over the SMs (one tile each) when that is
+    // under 128 rows, at least 16
+    const int64_t share = (a.T + sm_count() - 1) / sm_count();
+    p.tile_rows = (int)std::max<int64_t>(16, std::min<int64_t>(BM, share));
     CUtensorMap ma, mb;
-    if (!make_map(&ma, a.x, a.d, a.T, BM)) return cudaErrorInvalidValue;
+    if (!make_map(&ma, a.x, a.d, a.T, p.tile_rows)) return cudaErrorInvalidValue;
     if (!make_map(&mb, a.w_router, a.d, (int64_t)a.P * a.E, BNr)) return cudaErrorInvalidValue;
-    const int64_t tiles = (a.T + BM - 1) / BM + a.P;
+    const int64_t tiles = (a.T + p.tile_rows - 1) / p.tile_rows + a.P;
     if (BNr == 16) return launch<16, false, false, EPI_ROUTE>(ma, mb, ma, ma, p, tiles, s);
     if (BNr == 32) return launch<32, false, false, EPI_ROUTE>(ma, mb, ma, ma, p, tiles, s);
     if (BNr == 64) return launch<64, false, false, EPI_ROUTE>(ma, mb, ma, ma, p, tiles, s);
