@@ -77,7 +77,8 @@ def peaks():
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
             p = json.load(f)
         return {"hbm_gbs": p["hbm_gbs"], "bf16_tflops": p["bf16_tflops"],
-                "bf16_tflops_sustained": p.get("bf16_tflops_sustained"), "source": "measured"}
+                "bf16_tflops_sustained": p.get("bf16_tflops_sustained"), "source": "measured",
+                "sustained_sm_mhz": (p.get("clocks_under_load") or {}).get("sm_mhz_median")}
     except Exception:
         return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
                 "source": "fallback"}
@@ -532,6 +533,7 @@ def main():
                 "frac": achieved / pk["bf16_tflops"], "traffic": traffic,
                 "peak_source": f"{pk['source']} bf16 burst (torch.matmul 8192^3, best of 10)",
                 "peak_sustained": pk["bf16_tflops_sustained"],
+                "peak_sustained_sm_mhz": pk.get("sustained_sm_mhz"),
                 "frac_sustained": (achieved / pk["bf16_tflops_sustained"]
                                    if pk["bf16_tflops_sustained"] else None),
                 "peak_nominal": NOMINAL_BF16_TFLOPS,
