@@ -155,8 +155,10 @@ def test_training_calls_check_arguments_on_host(L):
 def test_backward_kernel_count_follows_the_tile_mode(L):
     """moe_expert_ffn_bwd_kernels (host only): in the default mode the dA GEMM shares a
     launch with dW2 and dX runs as CTA pairs beside a separate dW1 launch (3); with
-    single-CTA tiles both pairs of GEMMs share launches (2); fp32 runs four; shared
-    experts add four; nothing to do, no GEMM."""
+    single-CTA tiles both pairs of GEMMs share launches (2); fp32 runs four; with
+    d = 2048 and F = 1408 every backward GEMM of the routed and the shared experts runs as
+    its own pair launch (dA and dX as pairs with a ragged last N-tile, 8); nothing to do,
+    no GEMM."""
     mid = L.make_config(4096, 1024, 16, 2816, 2)
     assert L.moe_expert_ffn_bwd_kernels(mid) == 3
     try:
@@ -168,7 +170,7 @@ def test_backward_kernel_count_follows_the_tile_mode(L):
         L.moe_set_gemm_pairs(L.MOE_PAIRS_AUTO)
     assert L.moe_expert_ffn_bwd_kernels(L.make_config(512, 256, 8, 512, 2, dtype=L.MOE_F32)) == 4
     assert L.moe_expert_ffn_bwd_kernels(L.make_config(8192, 2048, 64, 1408, 6, n_shared=2,
-                                                      d_ff_shared=1408)) == 7
+                                                      d_ff_shared=1408)) == 8
     assert L.moe_expert_ffn_bwd_kernels(L.make_config(0, 1024, 16, 2816, 2)) == 0
 
 
