@@ -29,8 +29,12 @@ constexpr int BK = 64;  // 64 bf16 = 128 bytes = one 128B-swizzle row
 __host__ __device__ constexpr int kblock_rows(bool var_k, bool pair) { return (var_k && pair) ? 128 : BK; }
 // k-blocks per operand stage: 2 for the router up to 64 experts (its stream of x is bound
 // by a fixed cost per stage hand-off, so a stage carries two 64-wide boxes of each
-// operand; wider B would leave too few stages), else 1
-__host__ __device__ constexpr int kblocks_per_stage(int epi, int bn) { return (epi == 3 /* EPI_ROUTE */ && bn <= 64) ? 2 : 1; }
+// operand; wider B would leave too few stages) and for the M-variable CTA-pair tiles
+// (three stages of 64 KiB per CTA instead of six of 32: the same bytes in flight, half
+// the hand-offs, less power per flop under the power cap), else 1
+__host__ __device__ constexpr int kblocks_per_stage(int epi, int bn, bool pair = false, bool var_k = false) {
+    return ((epi == 3 /* EPI_ROUTE */ && bn <= 64) || (pair && !var_k)) ? 2 : 1;
+}
 constexpr int STAGES = 4;
 constexpr int EPI_WARPS = 4;
 constexpr int THREADS = 64 + 32 * EPI_WARPS;  // TMA warp, MMA warp, epilogue warps
@@ -549,7 +553,7 @@ __global__ void __launch_bounds__(THREADS, OCC)
     constexpr int BMP = BM * NPAIR;  // rows of one (pair) tile
     constexpr int KB = kblock_rows(VAR_K, PAIR);  // contraction rows per k-block
     constexpr uint32_t ATOM = KB * 128;              // bytes of one 64-wide MN-major box
-    constexpr int KPS = kblocks_per_stage(EPI, BN);
+    constexpr int KPS = kblocks_per_stage(EPI, BN, PAIR, VAR_K);
     constexpr uint32_t A_BOX = BM * KB * 2;   // one k-block of A
     constexpr uint32_t B_BOX = BNL * KB * 2;  // one k-block of B
     constexpr uint32_t A_BYTES = A_BOX * KPS;
@@ -859,7 +863,9 @@ __global__ void __launch_bounds__(THREADS, OCC)
                         // leader holds the gate half and the peer the up half
                         const int64_t r = (int64_t)ti.we * p.b_group_rows + ti.n0;
                         if constexpr (PAIR) {
-                            load(sb, &tmB, fb, k0, (int)(r + (rank ? p.F : 0)));
+#pragma unroll
+                            for (int j = 0; j < KPS; ++j)
+                                load(sb + j * B_BOX, &tmB, fb, k0 + KB * j, (int)(r + (rank ? p.F : 0)));
                         } else {
                             load(sb, &tmB, fb, k0, (int)r);
                             load(sb + 128 * 128, &tmB, fb, k0, (int)(r + p.F));
@@ -873,8 +879,11 @@ __global__ void __launch_bounds__(THREADS, OCC)
                         const int64_t krow = (VAR_K || dw) ? (ti.b_row + k0) : ((int64_t)ti.we * p.b_group_rows + k0);
                         const CUtensorMap* mB = dw ? &tmB2 : &tmB;
 #pragma unroll
-                        for (int i = 0; i < BNL / 64; ++i)
-                            load(sb + i * ATOM, mB, fb, ti.n0 + (int)rank * BNL + 64 * i, (int)krow);
+                        for (int j = 0; j < KPS; ++j)
+#pragma unroll
+                            for (int i = 0; i < BNL / 64; ++i)
+                                load(sb + j * B_BOX + i * ATOM, mB, fb, ti.n0 + (int)rank * BNL + 64 * i,
+                                     (int)(krow + KB * j));
                     }
                     issued_phase[stage] = (int)phase;
                     if (++stage == NST) {
@@ -960,9 +969,9 @@ __global__ void __launch_bounds__(THREADS, OCC)
                         if (kk >= ksteps) break;
                         uint64_t ad, bd;
                         if (!A_MN && !dwt) ad = smem_desc(sa + (kk / (KB / 16)) * A_BOX + (kk % (KB / 16)) * 32, 16, 1024);
-                        else ad = smem_desc(sa + kk * 2048, ATOM, 1024);
+                        else ad = smem_desc(sa + (kk / (KB / 16)) * A_BOX + (kk % (KB / 16)) * 2048, ATOM, 1024);
                         if (!B_MN) bd = smem_desc(sb + (kk / (KB / 16)) * B_BOX + (kk % (KB / 16)) * 32, 16, 1024);
-                        else bd = smem_desc(sb + kk * 2048, ATOM, 1024);
+                        else bd = smem_desc(sb + (kk / (KB / 16)) * B_BOX + (kk % (KB / 16)) * 2048, ATOM, 1024);
                         if constexpr (PAIR) mma_bf16_pair(tmem_d, ad, bd, IDESC, (kb | kk) ? 1u : 0u);
                         else mma_bf16(tmem_d, ad, bd, dwt ? IDESC_DW : IDESC, (kb | kk) ? 1u : 0u);
                     }
@@ -1377,7 +1386,7 @@ static cudaError_t launch(const CUtensorMap& ma, const CUtensorMap& mb, const CU
     Params P2 = p2 ? *p2 : p;
     constexpr int NPAIR = PAIR ? 2 : 1;
     constexpr int KB = kblock_rows(VAR_K, PAIR);
-    constexpr int STB = (BM * KB * 2 + BN / NPAIR * KB * 2) * kblocks_per_stage(EPI, BN);  // bytes of one operand stage
+    constexpr int STB = (BM * KB * 2 + BN / NPAIR * KB * 2) * kblocks_per_stage(EPI, BN, PAIR, VAR_K);  // bytes of one operand stage
     constexpr int NST = num_stages((uint32_t)STB, EPI, OCC);
     const int extra_max = EPI == EPI_ROUTE ? 64 * 64 * 4 : EPI_WARPS * epi_stage_bytes(EPI);
     const int extra = EPI == EPI_ROUTE ? p.hist_n * 4 : EPI_WARPS * epi_stage_bytes(EPI);
