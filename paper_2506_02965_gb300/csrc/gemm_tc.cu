@@ -35,7 +35,6 @@ __host__ __device__ constexpr int kblock_rows(bool var_k, bool pair) { return (v
 __host__ __device__ constexpr int kblocks_per_stage(int epi, int bn, bool pair = false, bool var_k = false) {
     return ((epi == 3 /* EPI_ROUTE */ && bn <= 64) || (pair && !var_k)) ? 2 : 1;
 }
-constexpr int STAGES = 4;
 constexpr int EPI_WARPS = 4;
 constexpr int THREADS = 64 + 32 * EPI_WARPS;  // TMA warp, MMA warp, epilogue warps
 constexpr int EPI_BOX = 32;                     // TMA-store box: 32 columns x 32 rows (bf16)
