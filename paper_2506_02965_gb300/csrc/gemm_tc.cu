@@ -30,10 +30,11 @@ __host__ __device__ constexpr int kblock_rows(bool var_k, bool pair) { return (v
 // k-blocks per operand stage: 2 for the router up to 64 experts (its stream of x is bound
 // by a fixed cost per stage hand-off, so a stage carries two 64-wide boxes of each
 // operand; wider B would leave too few stages) and for the M-variable CTA-pair tiles
-// (three stages of 64 KiB per CTA instead of six of 32: the same bytes in flight, half
-// the hand-offs, less power per flop under the power cap), else 1
+// with a store or SwiGLU-forward epilogue (three stages of 64 KiB per CTA instead of six
+// of 32: the same bytes in flight, half the hand-offs, less power per flop under the
+// power cap), else 1 (the SwiGLU-backward pairs measured faster with six stages)
 __host__ __device__ constexpr int kblocks_per_stage(int epi, int bn, bool pair = false, bool var_k = false) {
-    return ((epi == 3 /* EPI_ROUTE */ && bn <= 64) || (pair && !var_k)) ? 2 : 1;
+    return ((epi == 3 /* EPI_ROUTE */ && bn <= 64) || (pair && !var_k && epi != 2 /* EPI_SWIGLU_BWD */)) ? 2 : 1;
 }
 constexpr int EPI_WARPS = 4;
 constexpr int THREADS = 64 + 32 * EPI_WARPS;  // TMA warp, MMA warp, epilogue warps
