@@ -192,7 +192,7 @@ class PartyExpertLayer:
         T, TK, Eo = tokens, tokens * k, len(self.experts)
         self.x, self.dout = z(T, d), z(T, d)
         self.w_router, self.router_bias = z(1, E, d), None
-        self.w1, self.w2 = z(max(Eo, 1), 2 * F, d), z(max(Eo, 1), d, F)
+        self.w1, self.w2 = z(Eo, 2 * F, d), z(Eo, d, F)  # empty for a party hosting no expert
         self.logits, self.probs = z(T, E, dtype=f32), z(T, E, dtype=f32)
         self.topk_idx, self.topk_w = z(T, k, dtype=i32), z(T, k, dtype=f32)
         self.counts = z(1, E, dtype=i32)

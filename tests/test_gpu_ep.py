@@ -70,7 +70,8 @@ class PartyTransport:
 
 
 @pytest.mark.parametrize("P,E,k,Tp,d,F,zipf", [(2, 4, 2, 256, 256, 256, 0.0), (3, 8, 2, 200, 128, 256, 0.0),
-                                                (4, 8, 3, 384, 256, 512, 1.2), (2, 16, 4, 320, 128, 128, 0.0)])
+                                                (4, 8, 3, 384, 256, 512, 1.2), (2, 16, 4, 320, 128, 128, 0.0),
+                                                (3, 2, 2, 128, 128, 128, 0.0)])  # party 2 hosts no expert
 def test_parties_on_gpu_kernels_match_single_gpu_layer(P, E, k, Tp, d, F, zipf):
     L = need_gpu()
     sh = mi.MoEShape("ep", P * Tp, d, E, F, k, "bf16", n_parties=P, zipf_s=zipf, seed=500 + P)
@@ -115,6 +116,7 @@ def test_parties_on_gpu_kernels_match_single_gpu_layer(P, E, k, Tp, d, F, zipf):
 
     cross = 0
     for r, p in enumerate(parties):
+        assert p.dw1.shape[0] == len(p.experts) and p.dw2.shape[0] == len(p.experts)
         rows = slice(po[r], po[r + 1])
         assert torch.equal(p.topk_idx, ref.topk_idx[rows])
         assert torch.equal(p.counts[0], ref.counts[r])
