@@ -65,7 +65,8 @@ def _rank_main(rank, P, E, k, Tp, seed, port, out_dir):
     idx = mo.topk_indices(z.astype(np.float32), k)
     w = mo.gate_weights(p, idx, sh.normalize_topk)
     cnt = mo.party_counts(idx, E, one)[0]
-    plan = ep.make_plan(ep.gather_counts(cnt), rank)
+    tr = ep.DistTransport()  # the GPU party layer's transport, here over gloo
+    plan = ep.make_plan(tr.gather_counts(cnt), rank)
     # rows grouped by host party (owner = e mod P): only this party's tokens
     po_local = np.array([0] * (rank + 1) + [Ts] * (P - rank))
     _, _, _, slot, tok, send = mo.owner_dispatch_tables(idx, E, po_local)
@@ -87,7 +88,7 @@ def _rank_main(rank, P, E, k, Tp, seed, port, out_dir):
     loss, coef = mo.aux_loss(p, cnt[None], one, k, sh.aux_alpha)
     # --- backward: output gradients to the hosts, input gradients back (Sec. 3.2)
     dy_perm, dw = mo.combine_backward(inp["dout"][rows], y_perm, w, slot)
-    dye = ep.exchange(torch.from_numpy(dy_perm), plan.send_splits, plan.recv_splits).numpy()[plan.to_expert]
+    dye = tr.exchange(torch.from_numpy(dy_perm), plan.send_splits, plan.recv_splits).numpy()[plan.to_expert]
     dxe = np.zeros((plan.rows_in, sh.d_model))
     dw1, dw2 = {}, {}
     for i, e in enumerate(plan.experts):
@@ -98,7 +99,7 @@ def _rank_main(rank, P, E, k, Tp, seed, port, out_dir):
             dxe[r], dw1[e], dw2[e] = dX, dW1, dW2
         else:
             dw1[e], dw2[e] = np.zeros((2 * F, sh.d_model)), np.zeros((sh.d_model, F))
-    dx_perm = ep.exchange(torch.from_numpy(dxe[plan.to_source]), plan.recv_splits,
+    dx_perm = tr.exchange(torch.from_numpy(dxe[plan.to_source]), plan.recv_splits,
                           plan.send_splits).numpy()
     loc = dict(x=x, w_router=inp["w_router"][rank:rank + 1], party_offsets=one)
     rb = mo.router_backward(loc, sh.with_(T=Ts, n_parties=1), p, idx, w, dw, coef)
